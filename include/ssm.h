@@ -1,0 +1,269 @@
+/*
+ * ssm.h -- C ABI of libssm: one structured-suffix (SSM) denoising step of a
+ * block-wise diffusion language model on an NVIDIA GB300 (sm_103a).
+ *
+ * The step (paper: "Accelerating Diffusion Language Models via Structured
+ * Suffix Modeling") has four stages, each one entry point here:
+ *   1. ssm_select_suffix      -- retained suffix positions R_t (Sec. 3.2, Eqs. 1-5)
+ *   2. ssm_build_step_input   -- sparse input X~_t = [P; B_t; R_t] with original
+ *                                positions and soft suffix embeddings (Eqs. 6-8)
+ *   3. ssm_attention          -- bidirectional MHA/GQA attention with rotary
+ *                                encodings at the original positions
+ *   4. ssm_unmask             -- vocabulary softmax, confidence, argmax and the
+ *                                threshold / top-k / margin commit (Sec. 4.1, 4.5)
+ *
+ * Conventions (all entry points):
+ *   - Every function returns ssm_status; nothing throws across the ABI.
+ *   - Pointers are DEVICE pointers unless the name starts with h_ (host).
+ *     The caller allocates and owns every buffer; the library allocates no
+ *     device memory.  Scratch memory, where a stage needs it, is a caller
+ *     buffer of at least the size the matching *_workspace_size() returns.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is the
+ *     legacy default stream).  Argument checks are synchronous, on the host:
+ *     a call that returns an error has enqueued nothing.
+ *   - Errors found on the device (an out-of-range token id, a wait that timed
+ *     out) do not stop the stream: the kernel writes zeros or skips the item
+ *     and records a code in a device error word; ssm_get_device_error()
+ *     synchronises the stream and returns (and clears) that code.
+ *   - Tensors are dense, row-major, with the innermost dimension last, in the
+ *     layouts given per argument.  bf16 data are IEEE bfloat16 bit patterns.
+ */
+#ifndef SSM_H_
+#define SSM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ssm_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  SSM_OK = 0,
+  SSM_ERR_INVALID_ARG = 1,  /* null pointer, negative size, budget, alpha outside [0,1] ... */
+  SSM_ERR_SHAPE = 2,        /* inconsistent shapes (G % B != 0, H_q % H_kv != 0 ...) */
+  SSM_ERR_CAPACITY = 3,     /* output or workspace smaller than required */
+  SSM_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
+  SSM_ERR_TIMEOUT = 5,      /* (device) a bounded wait inside a kernel expired */
+  SSM_ERR_UNSUPPORTED = 6,  /* valid but not implemented (head_dim not 64/128 ...) */
+  SSM_ERR_DEVICE_INPUT = 7  /* (device) an input value was out of range (token id >= vocab ...) */
+} ssm_status;
+
+typedef enum { SSM_DTYPE_BF16 = 0, SSM_DTYPE_F32 = 1 } ssm_dtype;
+
+typedef enum {
+  SSM_COMMIT_THRESHOLD = 0, /* "Par.": commit masked positions with confidence > threshold */
+  SSM_COMMIT_TOPK = 1,      /* "Vanilla" is topk = 1: the k most confident masked positions */
+  SSM_COMMIT_MARGIN = 2     /* commit masked positions with p1 - p2 > threshold */
+} ssm_commit_mode;
+
+const char* ssm_status_str(ssm_status s);
+const char* ssm_version(void);
+
+/* Synchronises `stream`, returns the first device-side error recorded by any
+ * libssm kernel since the last call (SSM_OK if none) and clears it. */
+ssm_status ssm_get_device_error(ssm_stream_t stream);
+
+/* Device-side wait limit, in nanoseconds, for every bounded spin inside the
+ * libssm kernels (default 2e9).  A wait that exceeds it records
+ * SSM_ERR_TIMEOUT and the kernel leaves the work item.  0 restores the default. */
+ssm_status ssm_set_wait_limit_ns(uint64_t ns);
+
+/* ------------------------------------------------------------------------- */
+/* 1. Structured suffix selection (Sec. 3.2 "Suffix Region Partition" Eq. 1,  */
+/*    "Suffix Token Retention" Eqs. 2-5).                                     */
+/* ------------------------------------------------------------------------- */
+
+/* Sequence layout: the prompt occupies positions [0, prompt_len); the
+ * generation [prompt_len, prompt_len + gen_len) is cut into gen_len/block_len
+ * blocks; block_idx is the block being decoded and the suffix is every later
+ * block.  Budgets are token counts:
+ *   local_budget  L: the first L suffix tokens are kept (Eq. 2; the paper's w
+ *                    blocks are L = w * block_len); if the whole suffix fits in
+ *                    L, every suffix token is kept;
+ *   middle_budget M: the start token of each middle block (Eq. 3), at most M
+ *                    of them (evenly strided, block q*nm/M, if there are more);
+ *   tail_budget   T: T evenly spaced tokens of the last block, start and end
+ *                    included (Eq. 4 is T = 2). */
+typedef struct {
+  int32_t prompt_len, gen_len, block_len, block_idx;
+  int32_t local_budget, middle_budget, tail_budget;
+} ssm_suffix_cfg;
+
+/* Host only, pure: region sizes of R_t for `cfg` (the three add up to |R_t|;
+ * h_n_tail counts tail tokens not already local).  Any output may be NULL. */
+ssm_status ssm_suffix_count(const ssm_suffix_cfg* cfg, int32_t* h_n_local, int32_t* h_n_mid,
+                            int32_t* h_n_tail);
+
+/* Writes R_t for `cfg` to positions[0 .. |R_t|) as ascending absolute int32
+ * positions, and |R_t| to *h_count (host).  capacity = length of `positions`;
+ * if capacity < |R_t| returns SSM_ERR_CAPACITY with *h_count set and enqueues
+ * nothing. */
+ssm_status ssm_select_suffix(const ssm_suffix_cfg* cfg, int32_t* positions, int32_t capacity,
+                             int32_t* h_count, ssm_stream_t stream);
+
+/* Several selections in one launch (e.g. sequences of a serving batch, each at
+ * its own block index).  h_cfgs: host array of n configs.  The sets are
+ * written back to back into `positions`; h_offsets (host, n + 1 entries) gets
+ * the start of each set and the total in h_offsets[n]. */
+ssm_status ssm_select_suffix_batch(const ssm_suffix_cfg* h_cfgs, int32_t n, int32_t* positions,
+                                   int64_t capacity, int64_t* h_offsets, ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 2. Sparse step input with soft suffix embeddings (Sec. 3.2 "Soft Suffix    */
+/*    Embedding Mixing" Eqs. 6-8, "Sparse Input Construction").               */
+/* ------------------------------------------------------------------------- */
+
+/* For every batch row b the output rows are
+ *   [0, n_prefix)                 x = E[prefix_tokens[b, j]]          (prompt, when recomputed)
+ *   [n_prefix, n_prefix+B)        x = E[block_tokens[b, j]]           (current block; a masked
+ *                                                                     position carries mask_id)
+ *   [n_prefix+B, n_prefix+B+R)    x = (1-alpha) E[mask_id] + alpha * sum_j p~_j E[ids_j]
+ * with p~_j = p_j / sum_j p_j over the previous step's top-k candidates of
+ * that suffix position (Eq. 6-8).  Candidates with id -1 are absent; a row with
+ * no candidate (or zero mass) is E[mask_id].  Sums are in fp32, the stored
+ * value is rounded to bf16 (nearest even).  pos_out gets the original absolute
+ * positions: 0..n_prefix-1, block_start..block_start+B-1, suffix_pos[0..R).
+ *
+ *   block_tokens   int32 [batch, block_len]
+ *   prefix_tokens  int32 [batch, n_prefix]             (NULL iff n_prefix == 0)
+ *   suffix_pos     int32 [n_suffix]                    (from ssm_select_suffix)
+ *   embed          bf16  [vocab, hidden]; hidden % 8 == 0, 16-byte aligned
+ *   prev_topk_ids  int32 [batch, n_suffix, k]          (NULL: no prediction anywhere)
+ *   prev_topk_prob fp32  [batch, n_suffix, k]          (previous-step probabilities)
+ *   x_out          bf16  [batch, n_prefix + block_len + n_suffix, hidden]
+ *   pos_out        int32 [n_prefix + block_len + n_suffix]   (may be NULL)
+ * 0 <= k <= 32, alpha in [0, 1].  A token id outside [0, vocab) (other than a
+ * -1 candidate) records SSM_ERR_DEVICE_INPUT and zeroes that row. */
+ssm_status ssm_build_step_input(const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                int32_t batch, int32_t n_prefix, int32_t block_len,
+                                int32_t block_start, const int32_t* suffix_pos, int32_t n_suffix,
+                                const void* embed, int64_t vocab, int32_t hidden, int32_t mask_id,
+                                const int32_t* prev_topk_ids, const float* prev_topk_prob,
+                                int32_t k, float alpha, void* x_out, int32_t* pos_out,
+                                ssm_stream_t stream);
+
+/* Ragged form: n_problems independent steps (one sequence each, e.g. every
+ * block index of a sweep, or a serving batch at mixed block indices) in one
+ * launch.  problems is a DEVICE array; problem p reads
+ *   block_tokens[block_tok_off .. + block_len), prefix_tokens[prefix_tok_off .. + n_prefix),
+ *   suffix_pos[suffix_off .. + n_suffix), prev_topk_*[(suffix_off)*k .. + n_suffix*k)
+ * and writes rows out_row .. out_row + n_prefix + block_len + n_suffix of
+ * x_out [*, hidden] and the same entries of pos_out.  max_rows bounds
+ * n_prefix + block_len + n_suffix over all problems (grid size). */
+typedef struct {
+  int64_t block_tok_off;
+  int64_t prefix_tok_off;
+  int64_t suffix_off;
+  int64_t out_row;
+  int32_t n_prefix;
+  int32_t n_suffix;
+  int32_t block_start;
+  int32_t reserved;
+} ssm_step_problem;
+
+ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t n_problems,
+                                       int32_t max_rows, int32_t block_len,
+                                       const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                       const int32_t* suffix_pos, const void* embed,
+                                       int64_t vocab, int32_t hidden, int32_t mask_id,
+                                       const int32_t* prev_topk_ids, const float* prev_topk_prob,
+                                       int32_t k, float alpha, void* x_out, int32_t* pos_out,
+                                       ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 3. Bidirectional attention over prefix cache + block + retained suffix     */
+/*    (Sec. 1 and Sec. 2: DLM attention is bidirectional; Sec. 3.2 "Sparse    */
+/*    Input Construction": retained tokens keep their original rotary         */
+/*    encodings; Table 4: prefix cache "PC.").                                 */
+/* ------------------------------------------------------------------------- */
+
+/* O = softmax(scale * Q^ K^T) V with no mask, per (batch, query head h), over
+ * keys [cache rows; new rows].  Q^ = RoPE(q, pos), new keys are RoPE(k_new,
+ * pos); cached keys are used as given (already rotated at their own positions).
+ * RoPE: rotate-half pairs (i, i + d/2), angle pos * theta^(-2i/d); theta == 0
+ * disables it.  GQA: query head h reads key/value head h / (h_q / h_kv).
+ * bf16 inputs, fp32 accumulation (tcgen05 tensor cores), bf16 output.
+ *
+ *   q            bf16 [batch, n_new, h_q, d]
+ *   k_new, v_new bf16 [batch, n_new, h_kv, d]    (the same rows as q)
+ *   pos          int32 [n_new]                   (shared by the batch)
+ *   k_cache, v_cache bf16 [batch, n_cache, h_kv, d]  (NULL iff n_cache == 0)
+ *   out          bf16 [batch, n_new, h_q, d]
+ *   lse          fp32 [batch, n_new, h_q]  natural-log sum-exp of the scaled
+ *                scores (may be NULL)
+ *   workspace    >= ssm_attention_workspace_size(batch * n_new, h_q, h_kv, d)
+ *                bytes, 256-byte aligned; holds the rotated queries and keys.
+ * d in {64, 128}; h_q % h_kv == 0; every pointer 16-byte aligned. */
+size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv,
+                                    int32_t head_dim);
+
+ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
+                         const void* k_cache, const void* v_cache, int32_t batch, int32_t n_new,
+                         int32_t n_cache, int32_t h_q, int32_t h_kv, int32_t head_dim,
+                         float rope_theta, float scale, void* out, float* lse, void* workspace,
+                         size_t ws_bytes, ssm_stream_t stream);
+
+/* Ragged form: independent problems packed along the row dimension.
+ * problems is a DEVICE array; problem p owns rows new_row .. new_row + n_new
+ * of q / k_new / v_new / out / lse / pos (packed [total_new_rows, h, d]) and
+ * rows cache_row .. cache_row + n_cache of k_cache / v_cache (packed
+ * [total_cache_rows, h_kv, d]; several problems may share cache rows).
+ * max_n_new / max_n_cache bound the per-problem sizes (grid size).  A tile at
+ * the ragged end of a problem may read rows of the same buffers beyond it
+ * (multiplied by an exact zero): keep every row of the packed buffers finite. */
+typedef struct {
+  int64_t new_row;
+  int64_t cache_row;
+  int32_t n_new;
+  int32_t n_cache;
+} ssm_attn_problem;
+
+ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_new,
+                                const int32_t* pos, const void* k_cache, const void* v_cache,
+                                int64_t total_new_rows, int64_t total_cache_rows,
+                                const ssm_attn_problem* problems, int32_t n_problems,
+                                int32_t max_n_new, int32_t max_n_cache, int32_t h_q,
+                                int32_t h_kv, int32_t head_dim, float rope_theta, float scale,
+                                void* out, float* lse, void* workspace, size_t ws_bytes,
+                                ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 4. Confidence-based unmasking (Sec. 4.1 "Baselines": Vanilla top-1 and     */
+/*    parallel threshold decoding; Sec. 4.5: margin decoding).                */
+/* ------------------------------------------------------------------------- */
+
+/* For every masked block position (masked[b, j] != 0): the softmax over the
+ * vocabulary in fp32, conf = largest probability, argmax = lowest id among the
+ * largest logits, p2 = second-largest probability (a tied maximum counts
+ * twice).  Unmasked positions get conf = 0, argmax = -1, p2 = 0, commit = 0
+ * and their logits are never read.  Then, per batch row:
+ *   THRESHOLD: commit masked positions with conf > threshold;
+ *   MARGIN:    commit masked positions with conf - p2 > threshold;
+ *   TOPK:      commit the `topk` masked positions of highest confidence;
+ * and (THRESHOLD, MARGIN) if fewer than min_commit passed, the most confident
+ * remaining masked positions are added up to min_commit.  Ties between
+ * positions go to the lower position.
+ *
+ *   logits   [batch, block_len, vocab] of `dtype` (bf16 or fp32), 16-byte aligned
+ *   masked   uint8 [batch, block_len]
+ *   conf, p2 fp32 [batch, block_len]; argmax int32 [batch, block_len]
+ *            (p2 may be NULL unless mode == MARGIN)
+ *   commit   uint8 [batch, block_len]
+ *   workspace >= ssm_unmask_workspace_size(batch, block_len, vocab, dtype) bytes,
+ *            256-byte aligned (per-chunk partial reductions).
+ * block_len <= 1024. */
+size_t ssm_unmask_workspace_size(int32_t batch, int32_t block_len, int64_t vocab, ssm_dtype dtype);
+
+ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len,
+                      int64_t vocab, const uint8_t* masked, ssm_commit_mode mode, float threshold,
+                      int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
+                      uint8_t* commit, void* workspace, size_t ws_bytes, ssm_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SSM_H_ */

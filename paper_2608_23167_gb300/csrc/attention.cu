@@ -1,0 +1,669 @@
+// attention.cu -- bidirectional MHA/GQA attention over prefix cache + current
+// block + retained suffix (Sec. 1 and Sec. 2: DLM attention is non-causal;
+// Sec. 3.2 "Sparse Input Construction": retained suffix tokens keep their
+// original rotary encodings; Table 4 "PC.": prefix K/V come from a cache).
+//
+// Two kernels:
+//  * rope_pack_kernel rotates the new queries and keys at their original
+//    positions (fp64 angles, fp32 rotation, bf16 store) and packs the queries
+//    of one GQA group into one row block, (query i, head-in-group hl) -> row
+//    i * grp + hl, so that a 128-row M tile of the tensor-core GEMM is filled
+//    with every query head that shares a key/value head.
+//  * attn_fwd_kernel: one CTA per (problem, kv head, 128-row query tile).
+//    Warp 0 streams K/V tiles with TMA (128 keys = four 32-row sub-boxes, so
+//    the cache segment and the new-row segment pack back to back with at most
+//    31 padded keys each); warp 1 issues tcgen05.mma (S = Q K^T and O += P V,
+//    bf16 operands from shared memory, fp32 accumulators in tensor memory);
+//    warps 2-5 run the online softmax, one query row per thread, reading S
+//    from tensor memory and writing P (bf16) to shared memory.  S is double
+//    buffered in tensor memory so QK^T of tile j+1 overlaps the softmax of
+//    tile j.  O is rescaled only when a row maximum grows by more than 2^8.
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <mutex>
+
+#include "common.cuh"
+#include "sm100_ptx.cuh"
+#include "tmem_io.cuh"
+
+namespace ssm {
+namespace {
+
+constexpr int kBM = 128;            // query rows per tile (tcgen05 M)
+constexpr int kBN = 128;            // keys per tile (tcgen05 N of QK^T, K of PV)
+constexpr int kSub = 32;            // rows per TMA sub-box of a key tile
+constexpr int kAttnThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: softmax
+constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kOCol = 256;       // O accumulator columns; S buffers at 0 and 128
+constexpr uint64_t kDrainNs = 200000000ull;
+
+enum Bar {
+  Q_FULL = 0,
+  K_FULL = 1,   // [2]
+  K_EMPTY = 3,  // [2]
+  V_FULL = 5,   // [2]
+  V_EMPTY = 7,  // [2]
+  S_FULL = 9,   // [2]
+  S_FREE = 11,  // [2]
+  P_FULL = 13,  // [2]
+  P_FREE = 15,  // [2]
+  O_DONE = 17,
+  DRAIN = 18,
+  N_BARS = 19
+};
+
+template <int D>
+struct Layout {
+  static constexpr int NP = D / 64;                 // 64-column panels per row
+  static constexpr int Q = 0;
+  static constexpr int K = Q + NP * kPanel;         // 2 stages
+  static constexpr int V = K + 2 * NP * kPanel;     // 2 stages
+  static constexpr int P = V + 2 * NP * kPanel;     // 2 buffers of 128 x 128 bf16
+  static constexpr int BAR = P + 2 * 2 * kPanel;
+  static constexpr int BYTES = BAR + N_BARS * 8 + 8;
+  static constexpr int ALLOC = BYTES + 1024;        // slack to align the base to 1024 B
+  static_assert(ALLOC <= 232448, "shared memory budget");
+};
+
+struct AttnParams {
+  const ssm_attn_problem* problems;  // null: uniform batch
+  int32_t n_new_u, n_cache_u;
+  int32_t h_q, h_kv, grp;
+  int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
+  float scale_log2;                  // softmax scale * log2(e)
+  __nv_bfloat16* out;
+  float* lse;
+  unsigned* err;
+  uint64_t wait_ns;
+};
+
+struct Geom {
+  int64_t new_row, cache_row;
+  int32_t n_new, n_cache;
+};
+
+__device__ __forceinline__ Geom problem_geom(const AttnParams& p, int prob) {
+  Geom g;
+  if (p.problems) {
+    const ssm_attn_problem q = p.problems[prob];
+    g.new_row = q.new_row;
+    g.cache_row = q.cache_row;
+    g.n_new = q.n_new;
+    g.n_cache = q.n_cache;
+  } else {
+    g.n_new = p.n_new_u;
+    g.n_cache = p.n_cache_u;
+    g.new_row = static_cast<int64_t>(prob) * p.n_new_u;
+    g.cache_row = 0;
+  }
+  return g;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// ---------------------------------------------------------------------------
+// RoPE + GQA packing of the new rows
+// ---------------------------------------------------------------------------
+
+template <int D>
+__global__ void __launch_bounds__(128) rope_pack_kernel(
+    const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
+    const int32_t* __restrict__ pos, AttnParams p, float theta, __nv_bfloat16* __restrict__ qhat,
+    __nv_bfloat16* __restrict__ khat) {
+  constexpr int PPL = D / 64;  // rotation pairs per lane
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int prob = blockIdx.y;
+  const Geom gm = problem_geom(p, prob);
+  const int i = blockIdx.x * 4 + warp;
+  if (i >= gm.n_new) return;
+  const int32_t ps = pos[p.problems ? gm.new_row + i : i];
+  float cs[PPL], sn[PPL];
+#pragma unroll
+  for (int t = 0; t < PPL; ++t) {
+    if (theta > 0.f) {
+      const int jp = lane * PPL + t;
+      const double inv = pow(static_cast<double>(theta), -2.0 * jp / D);
+      double s, c;
+      sincos(static_cast<double>(ps) * inv, &s, &c);
+      cs[t] = static_cast<float>(c);
+      sn[t] = static_cast<float>(s);
+    } else {
+      cs[t] = 1.f;
+      sn[t] = 0.f;
+    }
+  }
+  auto rotate = [&](const __nv_bfloat16* src, __nv_bfloat16* dst) {
+    float x1[PPL], x2[PPL];
+    if constexpr (PPL == 2) {
+      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(src + 2 * lane);
+      const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(src + D / 2 + 2 * lane);
+      x1[0] = __low2float(a);
+      x1[1] = __high2float(a);
+      x2[0] = __low2float(b);
+      x2[1] = __high2float(b);
+    } else {
+      x1[0] = __bfloat162float(src[lane]);
+      x2[0] = __bfloat162float(src[D / 2 + lane]);
+    }
+    float y1[PPL], y2[PPL];
+#pragma unroll
+    for (int t = 0; t < PPL; ++t) {
+      y1[t] = x1[t] * cs[t] - x2[t] * sn[t];
+      y2[t] = x2[t] * cs[t] + x1[t] * sn[t];
+    }
+    if constexpr (PPL == 2) {
+      *reinterpret_cast<__nv_bfloat162*>(dst + 2 * lane) = __floats2bfloat162_rn(y1[0], y1[1]);
+      *reinterpret_cast<__nv_bfloat162*>(dst + D / 2 + 2 * lane) = __floats2bfloat162_rn(y2[0], y2[1]);
+    } else {
+      dst[lane] = __float2bfloat16_rn(y1[0]);
+      dst[D / 2 + lane] = __float2bfloat16_rn(y2[0]);
+    }
+  };
+  const int64_t row = gm.new_row + i;
+  for (int h = 0; h < p.h_q; ++h) {
+    const int g = h / p.grp, hl = h - g * p.grp;
+    const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
+                            static_cast<int64_t>(i) * p.grp + hl;
+    rotate(q + (row * p.h_q + h) * D, qhat + dst_row * D);
+  }
+  for (int g = 0; g < p.h_kv; ++g) rotate(k + (row * p.h_kv + g) * D, khat + (row * p.h_kv + g) * D);
+}
+
+// ---------------------------------------------------------------------------
+// Attention forward
+// ---------------------------------------------------------------------------
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
+    const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
+    const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kn,
+    const __grid_constant__ CUtensorMap tm_vn, const AttnParams p) {
+  using L = Layout<D>;
+  constexpr int NP = L::NP;
+  constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
+  constexpr uint32_t kIdescPV = idesc_bf16_f32(kBM, D, false, true);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + N_BARS);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int prob = blockIdx.y / p.h_kv;
+  const int g = blockIdx.y - prob * p.h_kv;
+  const int mt = blockIdx.x;
+  const Geom gm = problem_geom(p, prob);
+  const int rows_q = gm.n_new * p.grp;
+  if (mt * kBM >= rows_q) return;  // whole CTA, before any shared state exists
+  const bool uniform = p.problems == nullptr;
+  const int n_csub = (gm.n_cache + kSub - 1) / kSub;
+  const int n_nsub = (gm.n_new + kSub - 1) / kSub;
+  const int nt = (n_csub + n_nsub + 3) / 4;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars[Q_FULL], 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars[K_FULL + s], 1);
+      mbar_init(&bars[K_EMPTY + s], 1);
+      mbar_init(&bars[V_FULL + s], 1);
+      mbar_init(&bars[V_EMPTY + s], 1);
+      mbar_init(&bars[S_FULL + s], 1);
+      mbar_init(&bars[S_FREE + s], 128);
+      mbar_init(&bars[P_FULL + s], 128);
+      mbar_init(&bars[P_FREE + s], 1);
+    }
+    mbar_init(&bars[O_DONE], 1);
+    mbar_init(&bars[DRAIN], 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish_alloc_permit();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kc);
+    tma_prefetch_desc(&tm_vc);
+    tma_prefetch_desc(&tm_kn);
+    tma_prefetch_desc(&tm_vn);
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      bool ok = true;
+      int issued_k[2] = {0, 0}, issued_v[2] = {0, 0};
+      mbar_arrive_expect_tx(&bars[Q_FULL], NP * kPanel);
+      int qy, qz;
+      if (uniform) {
+        qy = mt * kBM;
+        qz = prob * p.h_kv + g;
+      } else {
+        qy = static_cast<int>((gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp) + mt * kBM;
+        qz = 0;
+      }
+#pragma unroll
+      for (int pn = 0; pn < NP; ++pn) tma_load_3d(smem + L::Q + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+      const int c3 = uniform ? prob : 0;
+      for (int j = 0; j < nt && ok; ++j) {
+        const int st = j & 1;
+        const uint32_t empty_par = ((j >> 1) - 1) & 1;
+        for (int half = 0; half < 2 && ok; ++half) {  // half 0: K, half 1: V
+          if (j >= 2) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], empty_par, p.wait_ns);
+          if (!ok) break;
+          uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
+          mbar_arrive_expect_tx(full, NP * kPanel);
+          uint8_t* dst = smem + (half ? L::V : L::K) + st * NP * kPanel;
+#pragma unroll
+          for (int sb = 0; sb < 4; ++sb) {
+            const int sub = 4 * j + sb;
+            const CUtensorMap* map;
+            int c2;
+            if (sub < n_csub) {
+              map = half ? &tm_vc : &tm_kc;
+              c2 = uniform ? sub * kSub : static_cast<int>(gm.cache_row + sub * kSub);
+            } else if (sub - n_csub < n_nsub) {
+              map = half ? &tm_vn : &tm_kn;
+              c2 = uniform ? (sub - n_csub) * kSub : static_cast<int>(gm.new_row + (sub - n_csub) * kSub);
+            } else {
+              map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
+              c2 = p.new_rows_extent;
+            }
+#pragma unroll
+            for (int pn = 0; pn < NP; ++pn)
+              tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, g, c2, c3);
+          }
+          if (half) ++issued_v[st];
+          else ++issued_k[st];
+        }
+      }
+      if (!ok) {
+        record_error(p.err, SSM_ERR_TIMEOUT);
+        // let every copy in flight land before the CTA's shared memory is released
+        mbar_wait(&bars[Q_FULL], 0, kDrainNs);
+        for (int s = 0; s < 2; ++s) {
+          if (issued_k[s]) mbar_wait(&bars[K_FULL + s], (issued_k[s] - 1) & 1, kDrainNs);
+          if (issued_v[s]) mbar_wait(&bars[V_FULL + s], (issued_v[s] - 1) & 1, kDrainNs);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(&bars[Q_FULL], 0, p.wait_ns);
+      tc_fence_after_sync();
+      const uint32_t sQ = smem_u32(smem + L::Q);
+      const uint32_t sK = smem_u32(smem + L::K);
+      const uint32_t sV = smem_u32(smem + L::V);
+      const uint32_t sP = smem_u32(smem + L::P);
+      for (int j = 0; j <= nt && ok; ++j) {
+        if (j < nt) {
+          const int sb = j & 1;
+          ok = mbar_wait(&bars[K_FULL + sb], (j >> 1) & 1, p.wait_ns);
+          if (ok && j >= 2) ok = mbar_wait(&bars[S_FREE + sb], ((j >> 1) - 1) & 1, p.wait_ns);
+          if (!ok) break;
+          tc_fence_after_sync();
+          const uint32_t kb = sK + sb * NP * kPanel;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
+            umma_bf16_ss(tmem + sb * kBN, sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024),
+                         kIdescQK, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(&bars[S_FULL + sb]);
+          umma_commit(&bars[K_EMPTY + sb]);
+        }
+        if (j >= 1) {
+          const int jj = j - 1, pb = jj & 1;
+          ok = mbar_wait(&bars[P_FULL + pb], (jj >> 1) & 1, p.wait_ns);
+          if (ok) ok = mbar_wait(&bars[V_FULL + pb], (jj >> 1) & 1, p.wait_ns);
+          if (!ok) break;
+          tc_fence_after_sync();
+          const uint32_t vb = sV + pb * NP * kPanel;
+          const uint32_t pbuf = sP + pb * 2 * kPanel;
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk) {
+            const uint64_t ad = sdesc_sw128(pbuf + (kk >> 2) * kPanel + (kk & 3) * 32, 16, 1024);
+            const uint64_t bd = sdesc_sw128(vb + kk * 16 * 128, kPanel, 1024);
+            umma_bf16_ss(tmem + kOCol, ad, bd, kIdescPV, (jj > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit(&bars[O_DONE]);
+          umma_commit(&bars[V_EMPTY + pb]);
+          umma_commit(&bars[P_FREE + pb]);
+        }
+      }
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+      // every issued MMA completes before tensor memory is released
+      umma_commit(&bars[DRAIN]);
+      mbar_wait(&bars[DRAIN], 0, kDrainNs);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------- softmax (warps 2..5)
+    const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31 belong to this warp
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t sP = smem_u32(smem + L::P);
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt; ++j) {
+      const int sb = j & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars[S_FULL + sb], (j >> 1) & 1, p.wait_ns));
+      if (!ok) break;
+      tc_fence_after_sync();
+      uint32_t sr[kBN];
+      tmem_ld_x128(tmem + lane_off + sb * kBN, sr);
+      tc_fence_before_sync();
+      mbar_arrive(&bars[S_FREE + sb]);
+
+      // keys past the end of a segment (cache or new rows) are masked out
+      int vcnt[4];
+      bool full = true;
+#pragma unroll
+      for (int s4 = 0; s4 < 4; ++s4) {
+        const int sub = 4 * j + s4;
+        int c;
+        if (sub < n_csub) c = min(kSub, gm.n_cache - sub * kSub);
+        else if (sub - n_csub < n_nsub) c = min(kSub, gm.n_new - (sub - n_csub) * kSub);
+        else c = 0;
+        vcnt[s4] = c;
+        full = full && (c == kSub);
+      }
+      if (!full) {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c)
+          if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
+      }
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, __uint_as_float(sr[c]));
+      const float m_new = fmaxf(m_run, mx * p.scale_log2);
+      const bool need = m_new > m_run + kRescaleLog2;
+      if (__any_sync(0xffffffffu, need)) {
+        const float alpha = need ? ex2_approx(m_run - m_new) : 1.f;
+        if (j > 0) {
+          ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE], (j - 1) & 1, p.wait_ns));
+          if (!ok) break;
+          tc_fence_after_sync();
+#pragma unroll
+          for (int ch = 0; ch < D / 32; ++ch) {
+            uint32_t o[32];
+            tmem_ld_x32(tmem + lane_off + kOCol + ch * 32, o);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+            tmem_st_x32(tmem + lane_off + kOCol + ch * 32, o);
+          }
+          tc_fence_before_sync();
+        }
+        if (need) {
+          l_run *= alpha;
+          m_run = m_new;
+        }
+      }
+      const float neg = -m_run;
+      float rs = 0.f;
+      uint32_t pk[kBN / 2];
+#pragma unroll
+      for (int c = 0; c < kBN / 2; ++c) {
+        const float a = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), p.scale_log2, neg));
+        const float b = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), p.scale_log2, neg));
+        rs += a + b;
+        pk[c] = pack_bf16x2(a, b);
+      }
+      l_run += rs;
+      if (j >= 2) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars[P_FREE + sb], ((j >> 1) - 1) & 1, p.wait_ns));
+        if (!ok) break;
+      }
+      const uint32_t prow = sP + sb * 2 * kPanel + row * 128;
+#pragma unroll
+      for (int ch = 0; ch < kBN / 8; ++ch) {
+        const int pn = ch >> 3, cc = ch & 7;
+        st_shared_v4(prow + pn * kPanel + ((cc ^ (row & 7)) << 4), pk[4 * ch], pk[4 * ch + 1],
+                     pk[4 * ch + 2], pk[4 * ch + 3]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(&bars[P_FULL + sb]);
+    }
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE], (nt - 1) & 1, p.wait_ns));
+    if (ok) {
+      tc_fence_after_sync();
+      const int pr = mt * kBM + row;  // packed (query, head-in-group) row
+      const bool valid = pr < rows_q;
+      const int qi = pr / p.grp;
+      const int h = g * p.grp + (pr - qi * p.grp);
+      const float inv = 1.f / l_run;
+      __nv_bfloat16* dst = p.out + ((gm.new_row + qi) * p.h_q + h) * D;
+#pragma unroll
+      for (int ch = 0; ch < D / 32; ++ch) {
+        uint32_t o[32];
+        tmem_ld_x32(tmem + lane_off + kOCol + ch * 32, o);
+        if (valid) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 w;
+            w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
+            w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
+            w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
+            w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
+            d4[v] = w;
+          }
+        }
+      }
+      if (valid && p.lse) p.lse[(gm.new_row + qi) * p.h_q + h] = (m_run + log2f(l_run)) * kLn2;
+    } else {
+      record_error(p.err, SSM_ERR_TIMEOUT);
+    }
+    tc_fence_before_sync();
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// bf16 tensor [d3][d2][d1][d0] (d0 innermost) with box (64, b1, b2, b3), 128-byte swizzle.
+bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint32_t* box) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t gdim[4], gstride[3];
+  cuuint32_t bdim[4], estr[4] = {1, 1, 1, 1};
+  uint64_t stride = 2;
+  for (int i = 0; i < rank; ++i) {
+    gdim[i] = dims[i];
+    bdim[i] = box[i];
+    if (i > 0) gstride[i - 1] = stride;
+    stride *= dims[i];
+  }
+  const CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), gdim, gstride, bdim,
+                        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int D>
+ssm_status launch_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
+                            const void* k_cache, const void* v_cache, bool uniform, int32_t batch_or_np,
+                            int64_t new_rows_per_b, int64_t cache_rows_per_b, int32_t max_n_new,
+                            const ssm_attn_problem* problems, int32_t h_q, int32_t h_kv,
+                            float rope_theta, float scale, void* out, float* lse, void* workspace,
+                            cudaStream_t st) {
+  using L = Layout<D>;
+  const int grp = h_q / h_kv;
+  const int64_t nb = uniform ? batch_or_np : 1;
+  const int64_t total_new = uniform ? static_cast<int64_t>(batch_or_np) * new_rows_per_b : new_rows_per_b;
+  auto* qhat = static_cast<__nv_bfloat16*>(workspace);
+  auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) +
+                                                align_up(static_cast<size_t>(total_new) * h_q * D * 2, 256));
+  CUtensorMap tq, tkc, tvc, tkn, tvn;
+  {
+    const uint64_t dq[3] = {static_cast<uint64_t>(D),
+                            static_cast<uint64_t>(uniform ? new_rows_per_b * grp : total_new * h_q),
+                            static_cast<uint64_t>(uniform ? nb * h_kv : 1)};
+    const uint32_t bq[3] = {64, kBM, 1};
+    if (!make_map(&tq, qhat, 3, dq, bq)) return SSM_ERR_CUDA;
+    const uint32_t bkv[4] = {64, 1, kSub, 1};
+    const uint64_t dn[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
+                            static_cast<uint64_t>(new_rows_per_b), static_cast<uint64_t>(nb)};
+    if (!make_map(&tkn, khat, 4, dn, bkv)) return SSM_ERR_CUDA;
+    if (!make_map(&tvn, v_new, 4, dn, bkv)) return SSM_ERR_CUDA;
+    if (cache_rows_per_b > 0) {
+      const uint64_t dc[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
+                              static_cast<uint64_t>(cache_rows_per_b), static_cast<uint64_t>(nb)};
+      if (!make_map(&tkc, k_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
+      if (!make_map(&tvc, v_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
+    } else {
+      tkc = tkn;  // never read: no problem has cache rows
+      tvc = tvn;
+    }
+  }
+  AttnParams p{};
+  p.problems = uniform ? nullptr : problems;
+  p.n_new_u = uniform ? static_cast<int32_t>(new_rows_per_b) : 0;
+  p.n_cache_u = uniform ? static_cast<int32_t>(cache_rows_per_b) : 0;
+  p.h_q = h_q;
+  p.h_kv = h_kv;
+  p.grp = grp;
+  p.new_rows_extent = static_cast<int32_t>(new_rows_per_b);
+  p.scale_log2 = scale * kLog2e;
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.lse = lse;
+  p.err = device_error_word();
+  p.wait_ns = wait_limit_ns();
+  const int n_prob = batch_or_np;
+  {
+    dim3 grid((max_n_new + 3) / 4, n_prob);
+    rope_pack_kernel<D><<<grid, 128, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
+                                               static_cast<const __nv_bfloat16*>(k_new), pos, p, rope_theta,
+                                               qhat, khat);
+    const ssm_status s = launch_status();
+    if (s != SSM_OK) return s;
+  }
+  // the dynamic shared-memory opt-in is a per-device function attribute
+  static std::atomic<uint64_t> attr_set{0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(attr_set.load() & bit)) {
+    if (cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
+        cudaSuccess)
+      return SSM_ERR_CUDA;
+    attr_set.fetch_or(bit);
+  }
+  const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
+  dim3 grid(m_tiles, n_prob * h_kv);
+  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(tq, tkc, tvc, tkn, tvn, p);
+  return launch_status();
+}
+
+ssm_status check_attn(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
+                      int32_t h_q, int32_t h_kv, int32_t head_dim, float scale, float theta, void* out,
+                      void* workspace) {
+  if (!q || !k_new || !v_new || !pos || !out || !workspace) return SSM_ERR_INVALID_ARG;
+  if (h_q <= 0 || h_kv <= 0) return SSM_ERR_INVALID_ARG;
+  if (h_q % h_kv != 0) return SSM_ERR_SHAPE;
+  if (head_dim != 64 && head_dim != 128) return SSM_ERR_UNSUPPORTED;
+  if (!(scale > 0.f) || !(theta >= 0.f)) return SSM_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out)) return SSM_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SSM_ERR_INVALID_ARG;
+  return SSM_OK;
+}
+
+}  // namespace
+}  // namespace ssm
+
+extern "C" {
+
+size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv, int32_t head_dim) {
+  if (total_new_rows <= 0 || h_q <= 0 || h_kv <= 0 || head_dim <= 0) return 0;
+  return ssm::align_up(static_cast<size_t>(total_new_rows) * h_q * head_dim * 2, 256) +
+         ssm::align_up(static_cast<size_t>(total_new_rows) * h_kv * head_dim * 2, 256);
+}
+
+ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
+                         const void* k_cache, const void* v_cache, int32_t batch, int32_t n_new,
+                         int32_t n_cache, int32_t h_q, int32_t h_kv, int32_t head_dim,
+                         float rope_theta, float scale, void* out, float* lse, void* workspace,
+                         size_t ws_bytes, ssm_stream_t stream) {
+  if (batch < 0 || n_new < 0 || n_cache < 0) return SSM_ERR_INVALID_ARG;
+  if (batch == 0 || n_new == 0) return SSM_OK;
+  ssm_status s = ssm::check_attn(q, k_new, v_new, pos, h_q, h_kv, head_dim, scale, rope_theta, out, workspace);
+  if (s != SSM_OK) return s;
+  if (n_cache > 0 && (!k_cache || !v_cache || !ssm::aligned16(k_cache) || !ssm::aligned16(v_cache)))
+    return SSM_ERR_INVALID_ARG;
+  if (ws_bytes < ssm_attention_workspace_size(static_cast<int64_t>(batch) * n_new, h_q, h_kv, head_dim))
+    return SSM_ERR_CAPACITY;
+  if (static_cast<int64_t>(batch) * h_kv > 65535) return SSM_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(n_new) * (h_q / h_kv) > INT32_MAX / 2) return SSM_ERR_UNSUPPORTED;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (head_dim == 128)
+    return ssm::launch_attention<128>(q, k_new, v_new, pos, k_cache, v_cache, true, batch, n_new, n_cache, n_new,
+                                      nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
+  return ssm::launch_attention<64>(q, k_new, v_new, pos, k_cache, v_cache, true, batch, n_new, n_cache, n_new,
+                                   nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
+}
+
+ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_new,
+                                const int32_t* pos, const void* k_cache, const void* v_cache,
+                                int64_t total_new_rows, int64_t total_cache_rows,
+                                const ssm_attn_problem* problems, int32_t n_problems,
+                                int32_t max_n_new, int32_t max_n_cache, int32_t h_q,
+                                int32_t h_kv, int32_t head_dim, float rope_theta, float scale,
+                                void* out, float* lse, void* workspace, size_t ws_bytes,
+                                ssm_stream_t stream) {
+  if (n_problems < 0 || total_new_rows < 0 || total_cache_rows < 0 || max_n_new < 0 || max_n_cache < 0)
+    return SSM_ERR_INVALID_ARG;
+  if (n_problems == 0 || total_new_rows == 0 || max_n_new == 0) return SSM_OK;
+  ssm_status s = ssm::check_attn(q, k_new, v_new, pos, h_q, h_kv, head_dim, scale, rope_theta, out, workspace);
+  if (s != SSM_OK) return s;
+  if (!problems) return SSM_ERR_INVALID_ARG;
+  if (total_cache_rows > 0 && (!k_cache || !v_cache || !ssm::aligned16(k_cache) || !ssm::aligned16(v_cache)))
+    return SSM_ERR_INVALID_ARG;
+  if (ws_bytes < ssm_attention_workspace_size(total_new_rows, h_q, h_kv, head_dim)) return SSM_ERR_CAPACITY;
+  if (static_cast<int64_t>(n_problems) * h_kv > 65535) return SSM_ERR_UNSUPPORTED;
+  if (total_new_rows * h_q > INT32_MAX / 2 || total_cache_rows > INT32_MAX / 2) return SSM_ERR_UNSUPPORTED;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (head_dim == 128)
+    return ssm::launch_attention<128>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
+                                      total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out,
+                                      lse, workspace, st);
+  return ssm::launch_attention<64>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
+                                   total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out, lse,
+                                   workspace, st);
+}
+
+}  // extern "C"

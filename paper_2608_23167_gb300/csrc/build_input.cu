@@ -1,0 +1,292 @@
+// build_input.cu -- sparse step input with soft suffix embeddings
+// (Sec. 3.2 "Soft Suffix Embedding Mixing", Eqs. 6-8, and "Sparse Input
+// Construction": X~_t = [P; B_t; R_t] keeping the original positions).
+//
+// One CTA per output row.  Prompt and block rows are embedding-row copies;
+// a retained suffix row reads the [MASK] row plus its k previous-step
+// candidate rows and writes (1-alpha) e_mask + alpha * sum_j p~_j e_j.  Every
+// access is a 16-byte vector (8 bf16 values), so a row of hidden 4096 is 512
+// coalesced vectors.  The work is a gather: HBM-bound, no tensor cores.
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+
+namespace ssm {
+namespace {
+
+constexpr int kBuildThreads = 128;
+constexpr int kMaxK = 32;
+
+struct BuildParams {
+  const ssm_step_problem* problems;  // null: uniform batch
+  int32_t n_problems;
+  // uniform description (problems == null)
+  int32_t u_n_prefix, u_n_suffix, u_block_start;
+  int32_t block_len;
+  const int32_t* block_tokens;
+  const int32_t* prefix_tokens;
+  const int32_t* suffix_pos;
+  const uint4* embed;        // [vocab, hidden/8] 16-byte vectors
+  int64_t vocab;
+  int32_t hvec;              // hidden / 8
+  int32_t mask_id;
+  const int32_t* topk_ids;
+  const float* topk_prob;
+  int32_t k;
+  float alpha;
+  uint4* x_out;
+  int32_t* pos_out;
+  unsigned* err;
+};
+
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void copy_row(const uint4* __restrict__ src, uint4* __restrict__ dst, int hvec) {
+  for (int v = threadIdx.x; v < hvec; v += kBuildThreads) dst[v] = __ldg(src + v);
+}
+
+__device__ __forceinline__ void zero_row(uint4* __restrict__ dst, int hvec) {
+  for (int v = threadIdx.x; v < hvec; v += kBuildThreads) dst[v] = make_uint4(0, 0, 0, 0);
+}
+
+__global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const BuildParams p) {
+  __shared__ int32_t s_ids[kMaxK];
+  __shared__ float s_w[kMaxK];
+  __shared__ int32_t s_n;
+  __shared__ int32_t s_bad;
+
+  const int prob = blockIdx.y;
+  const int r = blockIdx.x;
+  int64_t block_tok_off, prefix_tok_off, suffix_off, out_row;
+  int32_t n_prefix, n_suffix, block_start;
+  if (p.problems) {
+    const ssm_step_problem q = p.problems[prob];
+    block_tok_off = q.block_tok_off;
+    prefix_tok_off = q.prefix_tok_off;
+    suffix_off = q.suffix_off;
+    out_row = q.out_row;
+    n_prefix = q.n_prefix;
+    n_suffix = q.n_suffix;
+    block_start = q.block_start;
+  } else {
+    n_prefix = p.u_n_prefix;
+    n_suffix = p.u_n_suffix;
+    block_start = p.u_block_start;
+    block_tok_off = static_cast<int64_t>(prob) * p.block_len;
+    prefix_tok_off = static_cast<int64_t>(prob) * n_prefix;
+    suffix_off = 0;  // positions shared by the batch; top-k rows indexed below
+    out_row = static_cast<int64_t>(prob) * (n_prefix + p.block_len + n_suffix);
+  }
+  const int32_t rows = n_prefix + p.block_len + n_suffix;
+  if (r >= rows) return;
+  uint4* dst = p.x_out + (out_row + r) * p.hvec;
+
+  // original position id of this row (Sec. 3.2: retained tokens keep their positions)
+  if (threadIdx.x == 0 && p.pos_out && (p.problems || prob == 0)) {
+    int32_t pos;
+    if (r < n_prefix) pos = r;
+    else if (r < n_prefix + p.block_len) pos = block_start + (r - n_prefix);
+    else pos = p.suffix_pos[suffix_off + (r - n_prefix - p.block_len)];
+    p.pos_out[(p.problems ? out_row : 0) + r] = pos;
+  }
+
+  if (r < n_prefix + p.block_len) {
+    const int32_t tok = (r < n_prefix) ? p.prefix_tokens[prefix_tok_off + r]
+                                       : p.block_tokens[block_tok_off + (r - n_prefix)];
+    if (tok < 0 || tok >= p.vocab) {
+      if (threadIdx.x == 0) record_error(p.err, SSM_ERR_DEVICE_INPUT);
+      zero_row(dst, p.hvec);
+      return;
+    }
+    copy_row(p.embed + static_cast<int64_t>(tok) * p.hvec, dst, p.hvec);
+    return;
+  }
+
+  // retained suffix row i: Eq. 6 renormalisation, Eq. 7 soft embedding, Eq. 8 mix
+  const int64_t i = r - n_prefix - p.block_len;
+  const int64_t cand = p.problems ? (suffix_off + i) * p.k
+                                  : (static_cast<int64_t>(prob) * n_suffix + i) * p.k;
+  if (threadIdx.x == 0) {
+    int n = 0, bad = 0;
+    float z = 0.f;
+    if (p.topk_ids) {
+      for (int j = 0; j < p.k; ++j) {
+        const int32_t id = p.topk_ids[cand + j];
+        if (id == -1) continue;
+        if (id < 0 || id >= p.vocab) { bad = 1; continue; }
+        s_ids[n] = id;
+        s_w[n] = p.topk_prob[cand + j];
+        z += s_w[n];
+        ++n;
+      }
+    }
+    if (!(z > 0.f)) n = 0;                       // no prediction: the row keeps e_mask
+    const float scale = n ? p.alpha / z : 0.f;   // alpha * p_j / sum(p) = alpha * p~_j
+    for (int j = 0; j < n; ++j) s_w[j] *= scale;
+    s_n = n;
+    s_bad = bad;
+    if (bad) record_error(p.err, SSM_ERR_DEVICE_INPUT);
+  }
+  __syncthreads();
+  if (s_bad) {
+    zero_row(dst, p.hvec);
+    return;
+  }
+  const int n = s_n;
+  const uint4* e_mask = p.embed + static_cast<int64_t>(p.mask_id) * p.hvec;
+  if (n == 0) {
+    copy_row(e_mask, dst, p.hvec);
+    return;
+  }
+  const float keep = 1.f - p.alpha;
+  for (int v = threadIdx.x; v < p.hvec; v += kBuildThreads) {
+    float acc[8];
+    {
+      float m[8];
+      unpack8(__ldg(e_mask + v), m);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[c] = 0.f;
+      // gather the candidate rows four at a time so several loads are in flight
+      int j = 0;
+      for (; j + 4 <= n; j += 4) {
+        uint4 e4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) e4[u] = __ldg(p.embed + static_cast<int64_t>(s_ids[j + u]) * p.hvec + v);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          float f[8];
+          unpack8(e4[u], f);
+          const float w = s_w[j + u];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) acc[c] = fmaf(w, f[c], acc[c]);
+        }
+      }
+      for (; j < n; ++j) {
+        float f[8];
+        unpack8(__ldg(p.embed + static_cast<int64_t>(s_ids[j]) * p.hvec + v), f);
+        const float w = s_w[j];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) acc[c] = fmaf(w, f[c], acc[c]);
+      }
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[c] = fmaf(keep, m[c], acc[c]);
+    }
+    uint4 o;
+    o.x = pack2(acc[0], acc[1]);
+    o.y = pack2(acc[2], acc[3]);
+    o.z = pack2(acc[4], acc[5]);
+    o.w = pack2(acc[6], acc[7]);
+    dst[v] = o;
+  }
+}
+
+ssm_status check_common(const void* embed, int64_t vocab, int32_t hidden, int32_t mask_id, int32_t k,
+                        float alpha, int32_t block_len, const void* x_out) {
+  if (!embed || !x_out || vocab <= 0 || hidden <= 0 || block_len < 0) return SSM_ERR_INVALID_ARG;
+  if (hidden % 8 != 0) return SSM_ERR_UNSUPPORTED;
+  if (!aligned16(embed) || !aligned16(x_out)) return SSM_ERR_INVALID_ARG;
+  if (mask_id < 0 || mask_id >= vocab) return SSM_ERR_INVALID_ARG;
+  if (k < 0 || k > kMaxK) return SSM_ERR_UNSUPPORTED;
+  if (!(alpha >= 0.f && alpha <= 1.f)) return SSM_ERR_INVALID_ARG;
+  return SSM_OK;
+}
+
+}  // namespace
+}  // namespace ssm
+
+extern "C" {
+
+ssm_status ssm_build_step_input(const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                int32_t batch, int32_t n_prefix, int32_t block_len,
+                                int32_t block_start, const int32_t* suffix_pos, int32_t n_suffix,
+                                const void* embed, int64_t vocab, int32_t hidden, int32_t mask_id,
+                                const int32_t* prev_topk_ids, const float* prev_topk_prob,
+                                int32_t k, float alpha, void* x_out, int32_t* pos_out,
+                                ssm_stream_t stream) {
+  ssm_status s = ssm::check_common(embed, vocab, hidden, mask_id, k, alpha, block_len, x_out);
+  if (s != SSM_OK) return s;
+  if (batch < 0 || n_prefix < 0 || n_suffix < 0 || block_start < 0) return SSM_ERR_INVALID_ARG;
+  if (block_len > 0 && !block_tokens) return SSM_ERR_INVALID_ARG;
+  if (n_prefix > 0 && !prefix_tokens) return SSM_ERR_INVALID_ARG;
+  if (n_suffix > 0 && !suffix_pos) return SSM_ERR_INVALID_ARG;
+  if (prev_topk_ids && k > 0 && !prev_topk_prob) return SSM_ERR_INVALID_ARG;
+  const int32_t rows = n_prefix + block_len + n_suffix;
+  if (batch == 0 || rows == 0) return SSM_OK;
+  if (batch > 65535) return SSM_ERR_UNSUPPORTED;
+  ssm::BuildParams p{};
+  p.problems = nullptr;
+  p.n_problems = batch;
+  p.u_n_prefix = n_prefix;
+  p.u_n_suffix = n_suffix;
+  p.u_block_start = block_start;
+  p.block_len = block_len;
+  p.block_tokens = block_tokens;
+  p.prefix_tokens = prefix_tokens;
+  p.suffix_pos = suffix_pos;
+  p.embed = static_cast<const uint4*>(embed);
+  p.vocab = vocab;
+  p.hvec = hidden / 8;
+  p.mask_id = mask_id;
+  p.topk_ids = (k > 0) ? prev_topk_ids : nullptr;
+  p.topk_prob = prev_topk_prob;
+  p.k = k;
+  p.alpha = alpha;
+  p.x_out = static_cast<uint4*>(x_out);
+  p.pos_out = pos_out;
+  p.err = ssm::device_error_word();
+  dim3 grid(rows, batch);
+  ssm::build_step_input_kernel<<<grid, ssm::kBuildThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+  return ssm::launch_status();
+}
+
+ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t n_problems,
+                                       int32_t max_rows, int32_t block_len,
+                                       const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                       const int32_t* suffix_pos, const void* embed,
+                                       int64_t vocab, int32_t hidden, int32_t mask_id,
+                                       const int32_t* prev_topk_ids, const float* prev_topk_prob,
+                                       int32_t k, float alpha, void* x_out, int32_t* pos_out,
+                                       ssm_stream_t stream) {
+  ssm_status s = ssm::check_common(embed, vocab, hidden, mask_id, k, alpha, block_len, x_out);
+  if (s != SSM_OK) return s;
+  if (n_problems < 0 || max_rows < 0) return SSM_ERR_INVALID_ARG;
+  if (n_problems == 0 || max_rows == 0) return SSM_OK;
+  if (!problems || !suffix_pos || (block_len > 0 && !block_tokens)) return SSM_ERR_INVALID_ARG;
+  if (prev_topk_ids && k > 0 && !prev_topk_prob) return SSM_ERR_INVALID_ARG;
+  if (n_problems > 65535) return SSM_ERR_UNSUPPORTED;
+  ssm::BuildParams p{};
+  p.problems = problems;
+  p.n_problems = n_problems;
+  p.block_len = block_len;
+  p.block_tokens = block_tokens;
+  p.prefix_tokens = prefix_tokens;
+  p.suffix_pos = suffix_pos;
+  p.embed = static_cast<const uint4*>(embed);
+  p.vocab = vocab;
+  p.hvec = hidden / 8;
+  p.mask_id = mask_id;
+  p.topk_ids = (k > 0) ? prev_topk_ids : nullptr;
+  p.topk_prob = prev_topk_prob;
+  p.k = k;
+  p.alpha = alpha;
+  p.x_out = static_cast<uint4*>(x_out);
+  p.pos_out = pos_out;
+  p.err = ssm::device_error_word();
+  dim3 grid(max_rows, n_problems);
+  ssm::build_step_input_kernel<<<grid, ssm::kBuildThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+  return ssm::launch_status();
+}
+
+}  // extern "C"

@@ -1,0 +1,206 @@
+// select.cu -- structured suffix selection (Sec. 3.2, Eqs. 1-5).
+//
+// Each thread classifies suffix positions independently (a closed-form
+// membership test per position), and the CTA compacts the kept positions in
+// ascending order with warp ballots and a block-wide prefix sum.  One CTA per
+// selection; a batch of selections is one launch.
+#include <algorithm>
+#include <vector>
+
+#include "common.cuh"
+
+namespace ssm {
+namespace {
+
+// Closed-form description of R_t for one configuration (shared by the host
+// count and the device membership test).
+struct SuffixGeom {
+  int64_t s0;          // first suffix position
+  int64_t end;         // one past the last generated position
+  int64_t tail_start;  // first position of the tail block
+  int64_t mid_first;   // start position of the first middle block
+  int32_t B, L, M, T;
+  int32_t n_sb;        // number of suffix blocks
+  int32_t nm;          // number of middle blocks
+  bool all_local;
+};
+
+__host__ __device__ inline SuffixGeom make_geom(const ssm_suffix_cfg& c) {
+  SuffixGeom g{};
+  const int32_t nb = c.gen_len / c.block_len;
+  g.B = c.block_len;
+  g.L = c.local_budget;
+  g.M = c.middle_budget;
+  g.T = c.tail_budget;
+  g.s0 = static_cast<int64_t>(c.prompt_len) + static_cast<int64_t>(c.block_idx + 1) * c.block_len;
+  g.end = static_cast<int64_t>(c.prompt_len) + c.gen_len;
+  g.n_sb = nb - 1 - c.block_idx;
+  g.tail_start = static_cast<int64_t>(c.prompt_len) + static_cast<int64_t>(nb - 1) * c.block_len;
+  g.all_local = static_cast<int64_t>(g.n_sb) * g.B <= g.L;
+  // middle blocks: suffix blocks other than the tail whose start is >= s0 + L
+  const int64_t first = (static_cast<int64_t>(g.L) + g.B - 1) / g.B;  // blocks touched by local
+  g.mid_first = g.s0 + first * g.B;
+  const int64_t nm = static_cast<int64_t>(g.n_sb) - 1 - first;
+  g.nm = nm > 0 ? static_cast<int32_t>(nm) : 0;
+  return g;
+}
+
+__host__ __device__ inline int32_t tail_count(const SuffixGeom& g) {
+  return g.T >= g.B ? g.B : g.T;
+}
+
+// Is tail-block offset `o` one of the T evenly spaced offsets (j*(B-1))/(T-1)?
+__host__ __device__ inline bool tail_keeps(const SuffixGeom& g, int64_t o) {
+  if (g.T <= 0) return false;
+  if (g.T >= g.B) return true;
+  if (g.T == 1) return o == 0;
+  const int64_t num = o * (g.T - 1);
+  const int64_t j = (num + (g.B - 2)) / (g.B - 1);  // smallest j with j*(B-1)/(T-1) >= o
+  return j <= g.T - 1 && (j * (g.B - 1)) / (g.T - 1) == o;
+}
+
+// Is middle block number `mi` (0-based among middle blocks) one of the kept ones?
+__host__ __device__ inline bool middle_keeps(const SuffixGeom& g, int64_t mi) {
+  if (g.nm <= g.M) return true;
+  if (g.M <= 0) return false;
+  const int64_t q = (mi * g.M + g.nm - 1) / g.nm;  // smallest q with q*nm/M >= mi
+  return q < g.M && (q * g.nm) / g.M == mi;
+}
+
+__host__ __device__ inline bool keeps(const SuffixGeom& g, int64_t pos) {
+  if (g.all_local) return true;
+  if (pos < g.s0 + g.L) return true;                               // Eq. 2
+  if (pos >= g.tail_start) return tail_keeps(g, pos - g.tail_start);  // Eq. 4
+  if (pos >= g.mid_first && (pos - g.mid_first) % g.B == 0)         // Eq. 3
+    return middle_keeps(g, (pos - g.mid_first) / g.B);
+  return false;
+}
+
+void host_counts(const ssm_suffix_cfg& c, int32_t* nl, int32_t* nmid, int32_t* nt) {
+  const SuffixGeom g = make_geom(c);
+  if (g.n_sb <= 0) {
+    *nl = *nmid = *nt = 0;
+    return;
+  }
+  if (g.all_local) {
+    *nl = g.n_sb * g.B;
+    *nmid = *nt = 0;
+    return;
+  }
+  *nl = g.L;
+  *nmid = std::min(g.nm, g.M);
+  // tail tokens not already local
+  int32_t t = 0;
+  for (int64_t o = 0; o < g.B; ++o)
+    if (g.tail_start + o >= g.s0 + g.L && tail_keeps(g, o)) ++t;
+  *nt = t;
+}
+
+ssm_status check_cfg(const ssm_suffix_cfg* c) {
+  if (!c) return SSM_ERR_INVALID_ARG;
+  if (c->block_len <= 0 || c->gen_len <= 0 || c->prompt_len < 0) return SSM_ERR_INVALID_ARG;
+  if (c->gen_len % c->block_len != 0) return SSM_ERR_SHAPE;
+  if (c->block_idx < 0 || c->block_idx >= c->gen_len / c->block_len) return SSM_ERR_INVALID_ARG;
+  if (c->local_budget < 0 || c->middle_budget < 0 || c->tail_budget < 0) return SSM_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(c->prompt_len) + c->gen_len > INT32_MAX) return SSM_ERR_INVALID_ARG;
+  return SSM_OK;
+}
+
+constexpr int kSelThreads = 256;
+constexpr int kSelMaxPerLaunch = 64;  // keeps the kernel parameter block under 4 KB
+
+struct SelectBatch {
+  ssm_suffix_cfg cfg[kSelMaxPerLaunch];
+  int64_t offset[kSelMaxPerLaunch];
+};
+
+__global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectBatch batch,
+                                                             int32_t* __restrict__ positions) {
+  __shared__ int32_t warp_tot[kSelThreads / 32];
+  __shared__ int32_t base_s;
+  const ssm_suffix_cfg cfg = batch.cfg[blockIdx.x];
+  int32_t* out = positions + batch.offset[blockIdx.x];
+  const SuffixGeom g = make_geom(cfg);
+  if (g.n_sb <= 0) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) base_s = 0;
+  __syncthreads();
+  for (int64_t start = g.s0; start < g.end; start += kSelThreads) {
+    const int64_t pos = start + threadIdx.x;
+    const bool k = pos < g.end && keeps(g, pos);
+    const unsigned bal = __ballot_sync(0xffffffffu, k);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    int32_t before = 0, total = 0;
+#pragma unroll
+    for (int w = 0; w < kSelThreads / 32; ++w) {
+      before += (w < warp) ? warp_tot[w] : 0;
+      total += warp_tot[w];
+    }
+    const int32_t base = base_s;
+    if (k) out[base + before + __popc(bal & ((1u << lane) - 1u))] = static_cast<int32_t>(pos);
+    __syncthreads();
+    if (threadIdx.x == 0) base_s = base + total;
+    __syncthreads();
+  }
+}
+
+}  // namespace
+}  // namespace ssm
+
+extern "C" {
+
+ssm_status ssm_suffix_count(const ssm_suffix_cfg* cfg, int32_t* h_n_local, int32_t* h_n_mid,
+                            int32_t* h_n_tail) {
+  const ssm_status s = ssm::check_cfg(cfg);
+  if (s != SSM_OK) return s;
+  int32_t a, b, c;
+  ssm::host_counts(*cfg, &a, &b, &c);
+  if (h_n_local) *h_n_local = a;
+  if (h_n_mid) *h_n_mid = b;
+  if (h_n_tail) *h_n_tail = c;
+  return SSM_OK;
+}
+
+ssm_status ssm_select_suffix_batch(const ssm_suffix_cfg* h_cfgs, int32_t n, int32_t* positions,
+                                   int64_t capacity, int64_t* h_offsets, ssm_stream_t stream) {
+  if (n < 0 || (n > 0 && !h_cfgs) || capacity < 0) return SSM_ERR_INVALID_ARG;
+  std::vector<int64_t> off(static_cast<size_t>(n) + 1, 0);
+  for (int32_t i = 0; i < n; ++i) {
+    const ssm_status s = ssm::check_cfg(&h_cfgs[i]);
+    if (s != SSM_OK) return s;
+    int32_t a, b, c;
+    ssm::host_counts(h_cfgs[i], &a, &b, &c);
+    off[i + 1] = off[i] + a + b + c;
+  }
+  if (h_offsets)
+    for (int32_t i = 0; i <= n; ++i) h_offsets[i] = off[i];
+  if (off[n] > capacity) return SSM_ERR_CAPACITY;
+  if (off[n] > 0 && !positions) return SSM_ERR_INVALID_ARG;
+  for (int32_t first = 0; first < n; first += ssm::kSelMaxPerLaunch) {
+    const int32_t cnt = std::min(ssm::kSelMaxPerLaunch, n - first);
+    ssm::SelectBatch sb{};
+    for (int32_t i = 0; i < cnt; ++i) {
+      sb.cfg[i] = h_cfgs[first + i];
+      sb.offset[i] = off[first + i];
+    }
+    ssm::select_kernel<<<cnt, ssm::kSelThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(sb, positions);
+    const ssm_status ls = ssm::launch_status();
+    if (ls != SSM_OK) return ls;
+  }
+  return SSM_OK;
+}
+
+ssm_status ssm_select_suffix(const ssm_suffix_cfg* cfg, int32_t* positions, int32_t capacity,
+                             int32_t* h_count, ssm_stream_t stream) {
+  const ssm_status s = ssm::check_cfg(cfg);
+  if (s != SSM_OK) return s;
+  int32_t a, b, c;
+  ssm::host_counts(*cfg, &a, &b, &c);
+  if (h_count) *h_count = a + b + c;
+  if (capacity < a + b + c) return SSM_ERR_CAPACITY;
+  int64_t off[2];
+  return ssm_select_suffix_batch(cfg, 1, positions, capacity, off, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,90 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads, exports
+every entry point that include/ssm.h declares, and its pure host logic and
+argument validation behave as documented."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from oracle import ssm_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_23167_gb300 import build_lib, ssm
+    build_lib.build()
+    return ssm.lib()
+
+
+def _declared_functions():
+    with open(os.path.join(ROOT, "include", "ssm.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ssm_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = _declared_functions()
+    assert len(names) >= 14
+    for n in names:
+        assert hasattr(lib, n), n
+    from paper_2608_23167_gb300 import ssm
+    assert sorted(ssm.exported_symbols()) == names
+
+
+def test_status_strings_and_version(lib):
+    assert lib.ssm_status_str(0) == b"ok"
+    assert lib.ssm_status_str(3).startswith(b"output or workspace")
+    assert b"sm_103a" in lib.ssm_version()
+
+
+def test_suffix_count_matches_oracle(lib):
+    from paper_2608_23167_gb300 import ssm
+    for (P, G, B, L, M, T) in [(64, 256, 32, 32, 8, 4), (512, 1024, 32, 64, 32, 8), (1024, 2048, 32, 64, 64, 16),
+                               (0, 320, 32, 32, 3, 2), (16, 256, 32, 48, 1000, 2), (5, 96, 8, 12, 1, 9)]:
+        for b in range(G // B):
+            r, nl, nm, nt = O.select_suffix(P, G, B, b, L, M, T)
+            assert ssm.ssm_suffix_count(P, G, B, b, L, M, T) == (nl, nm, nt)
+
+
+def test_argument_validation_without_device(lib):
+    from paper_2608_23167_gb300 import ssm
+    cfg = ssm.SuffixCfg(0, 100, 32, 0, 32, 8, 4)          # G % B != 0
+    n = ctypes.c_int32()
+    assert lib.ssm_select_suffix(ctypes.byref(cfg), None, 0, ctypes.byref(n), None) == 2
+    cfg = ssm.SuffixCfg(0, 256, 32, 8, 32, 8, 4)          # block index out of range
+    assert lib.ssm_select_suffix(ctypes.byref(cfg), None, 0, ctypes.byref(n), None) == 1
+    cfg = ssm.SuffixCfg(64, 256, 32, 0, 32, 8, 4)         # capacity too small: count reported
+    assert lib.ssm_select_suffix(ctypes.byref(cfg), None, 10, ctypes.byref(n), None) == 3
+    assert n.value == 41
+    # attention: h_q % h_kv != 0, unsupported head_dim
+    fake = 1 << 20
+    assert lib.ssm_attention(fake, fake, fake, fake, None, None, 1, 8, 0, 6, 4, 128, 0.0, 0.1, fake, None,
+                             fake, 1 << 30, None) == 2
+    assert lib.ssm_attention(fake, fake, fake, fake, None, None, 1, 8, 0, 4, 4, 96, 0.0, 0.1, fake, None,
+                             fake, 1 << 30, None) == 6
+    assert lib.ssm_attention(fake, fake, fake, fake, None, None, 1, 8, 0, 4, 4, 128, 0.0, 0.1, fake, None,
+                             fake, 16, None) == 3
+    # unmask: bad dtype, block too long, workspace too small
+    assert lib.ssm_unmask(fake, 7, 1, 32, 4096, fake, 0, 0.9, 1, 1, fake, fake, fake, fake, fake, 1 << 20,
+                          None) == 6
+    assert lib.ssm_unmask(fake, 0, 1, 2048, 4096, fake, 0, 0.9, 1, 1, fake, fake, fake, fake, fake, 1 << 20,
+                          None) == 6
+    assert lib.ssm_unmask(fake, 0, 8, 32, 126464, fake, 0, 0.9, 1, 1, fake, fake, fake, fake, fake, 256,
+                          None) == 3
+    # build_step_input: alpha outside [0, 1], hidden not a multiple of 8
+    assert lib.ssm_build_step_input(fake, None, 1, 0, 32, 0, fake, 4, fake, 100, 64, 99, fake, fake, 5, 1.5,
+                                    fake, None, None) == 1
+    assert lib.ssm_build_step_input(fake, None, 1, 0, 32, 0, fake, 4, fake, 100, 60, 99, fake, fake, 5, 0.4,
+                                    fake, None, None) == 6
+
+
+def test_workspace_sizes(lib):
+    from paper_2608_23167_gb300 import ssm
+    import torch
+    assert ssm.ssm_attention_workspace_size(101 * 8, 32, 32, 128) == 2 * 101 * 8 * 32 * 128 * 2
+    ws = ssm.ssm_unmask_workspace_size(8, 32, 126464, torch.bfloat16)
+    assert ws >= 8 * 32 * 16 * 16 and ws % 256 == 0

@@ -1,0 +1,145 @@
+"""GPU parity: tcgen05 bidirectional attention against the fp64 oracle.
+
+Tolerance (attention): max-abs error <= 2e-2 and mean-abs error <= 2e-3 on the
+outputs; the natural-log LSE within 2e-2 absolute.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import ssm_oracle as O
+from paper_2608_23167_gb300 import workloads as W
+from tests.gpu_helpers import assert_attention_close, check_device_error, cuda_or_skip, f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def dev():
+    return cuda_or_skip()
+
+
+def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_lse=True):
+    from paper_2608_23167_gb300 import ssm
+    q = W.draw_normal_bf16((batch, n_new, h_q, d), 1.0, seed)
+    k = W.draw_normal_bf16((batch, n_new, h_kv, d), 1.0, seed + 1)
+    v = W.draw_normal_bf16((batch, n_new, h_kv, d), 1.0, seed + 2)
+    kc = W.draw_normal_bf16((batch, n_cache, h_kv, d), 1.0, seed + 3) if n_cache else None
+    vc = W.draw_normal_bf16((batch, n_cache, h_kv, d), 1.0, seed + 4) if n_cache else None
+    if pos is None:
+        g = torch.Generator().manual_seed(seed + 5)
+        pos = (n_cache + torch.randperm(4 * n_new + 7, generator=g)[:n_new]).to(torch.int32)
+    out = torch.full((batch, n_new, h_q, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    lse = torch.full((batch, n_new, h_q), float("nan"), dtype=torch.float32, device=dev) if with_lse else None
+    ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), None if kc is None else kc.to(dev),
+                      None if vc is None else vc.to(dev), out, theta, lse=lse)
+    torch.cuda.synchronize()
+    check_device_error()
+    ref, ref_lse = O.attention(f64(q), f64(k), f64(v), pos.numpy(), None if kc is None else f64(kc),
+                               None if vc is None else f64(vc), theta)
+    return f64(out), ref, (None if lse is None else f64(lse)), ref_lse
+
+
+@pytest.mark.parametrize("batch,n_new,n_cache,h_q,h_kv,d,theta", [
+    (1, 73, 64, 4, 4, 64, 1e4),          # tiny workload (b = 0)
+    (1, 589, 0, 8, 8, 128, 5e5),         # LLaDA no-cache shape (8 of 32 heads), 5 query tiles
+    (2, 132, 512, 14, 2, 128, 1e6),      # Dream GQA, 7 query heads per kv head
+    (2, 101, 512, 8, 8, 128, 5e5),       # serving shape (8 of 32 heads)
+    (1, 1, 0, 2, 1, 64, 1e4),            # a single key
+    (3, 37, 100, 4, 2, 128, 0.0),        # ragged cache (100 = 3*32 + 4), no rotary encoding
+    (1, 200, 1000, 2, 2, 64, 1e4),       # cache and new segments both ragged
+    (1, 129, 31, 4, 4, 128, 5e5),        # one row past a query tile
+])
+def test_attention_matches_oracle(dev, batch, n_new, n_cache, h_q, h_kv, d, theta):
+    out, ref, lse, ref_lse = _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache)
+    assert_attention_close(out, ref, f"b{batch} n{n_new} c{n_cache} h{h_q}/{h_kv} d{d}")
+    assert np.abs(lse - ref_lse).max() <= 2e-2
+
+
+def test_attention_full_workloads_sampled(dev):
+    """Full-size serving and Dream launches; the oracle checks a sample of heads."""
+    from paper_2608_23167_gb300 import ssm
+    for name in ("serve", "dream"):
+        w = W.WORKLOADS[name]
+        r, *_ = O.select_suffix(w.prompt, w.gen, w.block, 0, w.local, w.middle, w.tail)
+        n_new = w.block + len(r)
+        pos = torch.tensor(list(range(W.block_start(w, 0), W.block_start(w, 0) + w.block)) + r, dtype=torch.int32)
+        out, ref_unused, lse, _ = None, None, None, None
+        q = W.draw_normal_bf16((w.batch, n_new, w.h_q, w.head_dim), 1.0, 31)
+        k = W.draw_normal_bf16((w.batch, n_new, w.h_kv, w.head_dim), 1.0, 32)
+        v = W.draw_normal_bf16((w.batch, n_new, w.h_kv, w.head_dim), 1.0, 33)
+        kc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 34)
+        vc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 35)
+        o = torch.empty((w.batch, n_new, w.h_q, w.head_dim), dtype=torch.bfloat16, device=dev)
+        ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), o, w.rope_theta)
+        torch.cuda.synchronize()
+        check_device_error()
+        grp = w.h_q // w.h_kv
+        for b in (0, w.batch - 1):
+            g = w.h_kv - 1
+            hs = list(range(g * grp, (g + 1) * grp))
+            ref, _ = O.attention(f64(q[b:b + 1, :, hs]), f64(k[b:b + 1, :, g:g + 1]), f64(v[b:b + 1, :, g:g + 1]),
+                                 pos.numpy(), f64(kc[b:b + 1, :, g:g + 1]), f64(vc[b:b + 1, :, g:g + 1]),
+                                 w.rope_theta)
+            assert_attention_close(f64(o[b:b + 1, :, hs]), ref, f"{name} batch {b}")
+
+
+def test_attention_varlen_block_sweep(dev):
+    """The long-sequence sweep: every block index 0..63 as one ragged launch over a
+    shared prefix cache; the oracle checks several block indices on a few heads."""
+    from paper_2608_23167_gb300 import ssm
+    w = W.WORKLOADS["long"]
+    H, d = 4, w.head_dim                     # heads are independent in MHA: 4 of 32 suffice here
+    total_pos = w.prompt + w.gen
+    kc = W.draw_normal_bf16((total_pos, H, d), 1.0, 41)
+    vc = W.draw_normal_bf16((total_pos, H, d), 1.0, 42)
+    rows, poss, new_row = [], [], 0
+    for b in range(w.n_blocks):
+        r, *_ = O.select_suffix(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
+        bs = W.block_start(w, b)
+        p = list(range(bs, bs + w.block)) + r
+        rows.append((new_row, 0, len(p), bs))
+        poss.extend(p)
+        new_row += len(p)
+    q = W.draw_normal_bf16((new_row, H, d), 1.0, 43)
+    k = W.draw_normal_bf16((new_row, H, d), 1.0, 44)
+    v = W.draw_normal_bf16((new_row, H, d), 1.0, 45)
+    pos = torch.tensor(poss, dtype=torch.int32)
+    probs = ssm.attn_problems_tensor(rows, dev)
+    out = torch.full((new_row, H, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((new_row, H), dtype=torch.float32, device=dev)
+    ssm.ssm_attention_varlen(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), probs,
+                             len(rows), max(r[2] for r in rows), max(r[3] for r in rows), out, w.rope_theta,
+                             lse=lse)
+    torch.cuda.synchronize()
+    check_device_error()
+    og, lg = f64(out), f64(lse)
+    for b in (0, 1, 31, 43, 44, 60, 62, 63):
+        nr, _, n, nc = rows[b]
+        sl = slice(nr, nr + n)
+        ref, ref_lse = O.attention(f64(q[None, sl]), f64(k[None, sl]), f64(v[None, sl]), pos[sl].numpy(),
+                                   f64(kc[None, :nc]), f64(vc[None, :nc]), w.rope_theta)
+        assert_attention_close(og[sl][None], ref, f"block {b}")
+        assert np.abs(lg[sl][None] - ref_lse).max() <= 2e-2
+
+
+def test_attention_key_permutation_invariance(dev):
+    """Permuting the new rows together with their positions permutes the output rows."""
+    from paper_2608_23167_gb300 import ssm
+    n, c, h, d = 150, 70, 4, 128
+    q = W.draw_normal_bf16((1, n, h, d), 1.0, 51).to(dev)
+    k = W.draw_normal_bf16((1, n, h, d), 1.0, 52).to(dev)
+    v = W.draw_normal_bf16((1, n, h, d), 1.0, 53).to(dev)
+    kc = W.draw_normal_bf16((1, c, h, d), 1.0, 54).to(dev)
+    vc = W.draw_normal_bf16((1, c, h, d), 1.0, 55).to(dev)
+    pos = (c + torch.randperm(n)).to(torch.int32).to(dev)
+    perm = torch.randperm(n).to(dev)
+    o1 = torch.empty_like(q)
+    o2 = torch.empty_like(q)
+    ssm.ssm_attention(q, k, v, pos, kc, vc, o1, 1e4)
+    ssm.ssm_attention(q[:, perm].contiguous(), k[:, perm].contiguous(), v[:, perm].contiguous(),
+                      pos[perm].contiguous(), kc, vc, o2, 1e4)
+    torch.cuda.synchronize()
+    assert_attention_close(f64(o2), f64(o1[:, perm]), "permuted")
