@@ -1,0 +1,536 @@
+"""Benchmark of one structured-suffix (SSM) denoising pass on GB300.
+
+A bench step is one pass of the whole hot path -- suffix selection, sparse
+step input with soft suffix embeddings, bidirectional attention, unmasking --
+over one batch of synthetic input.  The default workload is the long-sequence
+LLaDA-8B shape (32 heads, head_dim 128, 1024-token prompt in a prefix cache,
+2048 generated tokens, block 32, budgets local 64 / middle 64 / tail 16) with
+every block index 0..63 decoded as one batch of 64 independent denoising
+steps, so one bench step = 64 denoising steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload long|serve|dream|llada|tiny]
+    python bench.py --impl reference ...   # the fp64 CPU oracle on the host cores
+
+Prints one JSON line (rank 0).  Multi-GPU runs (torchrun, one process per GPU)
+are independent replicas: the path has no exchange step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_23167_gb300 import workloads as W  # noqa: E402
+
+METRIC = "structured-suffix attn TFLOP/s (% bf16 peak); denoise steps/s; unmask HBM GB/s"
+UNIT = "denoise-steps/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ----------------------------------------------------------------------------- workload
+
+
+def suffix_positions(w: W.Workload, b: int):
+    """Host-side count of R_t from the library's pure host function (no device work)."""
+    from paper_2608_23167_gb300 import ssm
+    nl, nm, nt = ssm.ssm_suffix_count(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
+    return nl + nm + nt
+
+
+class StepInputs:
+    """Device-resident synthetic inputs of one bench step, plus the problem tables."""
+
+    def __init__(self, w: W.Workload, device, seed: int = 1234):
+        from paper_2608_23167_gb300 import ssm
+        self.w = w
+        self.dev = device
+        blocks = list(w.block_indices)
+        self.problems = [(s, b) for s in range(w.batch) for b in blocks]
+        n = len(self.problems)
+        self.n = n
+        self.cfgs = [(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail) for _, b in self.problems]
+        self.R = [suffix_positions(w, b) for _, b in self.problems]
+        n_prefix = 0 if w.prefix_cached else w.prompt
+        self.n_prefix = n_prefix
+        self.rows = [n_prefix + w.block + r for r in self.R]          # sparse-input rows per problem
+        self.row_off = np.concatenate([[0], np.cumsum(self.rows)]).astype(np.int64)
+        self.suf_off = np.concatenate([[0], np.cumsum(self.R)]).astype(np.int64)
+        self.total_rows = int(self.row_off[-1])
+        self.total_suffix = int(self.suf_off[-1])
+        V, H, k = w.vocab, w.hidden, w.topk
+        self.mask_id = V - 1
+        g = torch.Generator(device=device)
+        g.manual_seed(seed)
+        # model state: embedding table and (for the cached configurations) the prefix cache
+        self.embed = (torch.randn((V, H), generator=g, device=device) * 1.0).to(torch.bfloat16)
+        if w.prefix_cached:
+            if w.name == "long":
+                # one sequence: every block index reads the same cache, positions [0, prompt + b*B)
+                self.cache_rows = w.prompt + w.gen
+                self.cache_row = [0 for _ in self.problems]
+            else:
+                self.cache_rows = w.batch * w.prompt
+                self.cache_row = [s * w.prompt for s, _ in self.problems]
+            self.n_cache = [w.prompt + b * w.block for _, b in self.problems]
+            self.k_cache = torch.randn((self.cache_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
+            self.v_cache = torch.randn((self.cache_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
+        else:
+            self.cache_rows = 0
+            self.cache_row = [0] * n
+            self.n_cache = [0] * n
+            self.k_cache = self.v_cache = None
+        # per-step inputs: block tokens (first step of each block: all masked), previous-step
+        # top-k candidates, projections of the sparse input (stand-ins), LM-head logits (stand-ins)
+        self.block_tokens = torch.full((n, w.block), self.mask_id, dtype=torch.int32, device=device)
+        self.prefix_tokens = (torch.randint(0, V - 1, (n, n_prefix), generator=g, device=device, dtype=torch.int32)
+                              if n_prefix else None)
+        self.topk_ids = torch.randint(0, V - 1, (max(self.total_suffix, 1), k), generator=g, device=device,
+                                      dtype=torch.int32)
+        z = torch.softmax(torch.randn((max(self.total_suffix, 1), k), generator=g, device=device) * 3.0, dim=1)
+        self.topk_prob = (torch.sort(z, dim=1, descending=True).values *
+                          (0.2 + 0.8 * torch.rand((z.shape[0], 1), generator=g, device=device))).contiguous()
+        self.q = torch.randn((self.total_rows, w.h_q, w.head_dim), generator=g, device=device).to(torch.bfloat16)
+        self.k = torch.randn((self.total_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
+        self.v = torch.randn((self.total_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
+        lg = torch.randn((n, w.block, V), generator=g, device=device) * w.logits_sigma
+        self.logits = lg.to(torch.bfloat16) if w.logits_dtype == "bf16" else lg
+        del lg
+        self.masked = (self.block_tokens == self.mask_id).to(torch.uint8)
+        # outputs and scratch
+        self.positions = torch.zeros(max(self.total_suffix, 1), dtype=torch.int32, device=device)
+        self.x = torch.empty((self.total_rows, H), dtype=torch.bfloat16, device=device)
+        self.pos = torch.empty(self.total_rows, dtype=torch.int32, device=device)
+        self.out = torch.empty_like(self.q)
+        self.conf = torch.empty((n, w.block), dtype=torch.float32, device=device)
+        self.argmax = torch.empty((n, w.block), dtype=torch.int32, device=device)
+        self.p2 = torch.empty((n, w.block), dtype=torch.float32, device=device)
+        self.commit = torch.empty((n, w.block), dtype=torch.uint8, device=device)
+        self.attn_ws = torch.empty(ssm.ssm_attention_workspace_size(self.total_rows, w.h_q, w.h_kv, w.head_dim),
+                                   dtype=torch.uint8, device=device)
+        self.unmask_ws = torch.empty(ssm.ssm_unmask_workspace_size(n, w.block, V, self.logits.dtype),
+                                     dtype=torch.uint8, device=device)
+        self.step_tab = ssm.step_problems_tensor(
+            [(i * w.block, i * n_prefix, int(self.suf_off[i]), int(self.row_off[i]), n_prefix, self.R[i],
+              W.block_start(w, b)) for i, (_, b) in enumerate(self.problems)], device)
+        self.attn_tab = ssm.attn_problems_tensor(
+            [(int(self.row_off[i]), self.cache_row[i], self.rows[i], self.n_cache[i]) for i in range(n)], device)
+        self.max_rows = max(self.rows)
+        self.max_cache = max(self.n_cache)
+
+    # -- algorithmic work of one step ------------------------------------------------------
+    def attn_flops(self) -> float:
+        w = self.w
+        return float(sum(4.0 * w.h_q * w.head_dim * r * (r + c) for r, c in zip(self.rows, self.n_cache)))
+
+    def attn_bytes(self) -> float:
+        w = self.w
+        e = 2
+        qo = 2 * self.total_rows * w.h_q * w.head_dim * e
+        kv_new = 2 * self.total_rows * w.h_kv * w.head_dim * e
+        cache = 2 * (self.cache_rows if self.k_cache is not None else 0) * w.h_kv * w.head_dim * e
+        return float(qo + kv_new + cache)
+
+    def gather_bytes(self) -> float:
+        w = self.w
+        row = w.hidden * 2
+        reads = sum(self.n_prefix + w.block + w.topk * r for r in self.R) + 1       # + the [MASK] row
+        writes = self.total_rows
+        return float((reads + writes) * row)
+
+    def unmask_bytes(self) -> float:
+        w = self.w
+        masked_rows = int(self.masked.sum())
+        return float(masked_rows * w.vocab * self.logits.element_size())
+
+    # -- one pass of the hot path ---------------------------------------------------------
+    def step(self, ev=None):
+        from paper_2608_23167_gb300 import ssm
+        w = self.w
+        if ev is not None:
+            ev[0].record()
+        ssm.ssm_select_suffix_batch(self.positions, self.cfgs)
+        if ev is not None:
+            ev[1].record()
+        ssm.ssm_build_step_input_varlen(self.step_tab, self.n, self.max_rows, w.block, self.block_tokens,
+                                        self.positions, self.embed, self.mask_id, self.topk_ids, self.topk_prob,
+                                        w.topk, w.alpha, self.x, self.pos, prefix_tokens=self.prefix_tokens)
+        if ev is not None:
+            ev[2].record()
+        ssm.ssm_attention_varlen(self.q, self.k, self.v, self.pos, self.k_cache, self.v_cache, self.attn_tab,
+                                 self.n, self.max_rows, self.max_cache, self.out, w.rope_theta,
+                                 workspace=self.attn_ws)
+        if ev is not None:
+            ev[3].record()
+        ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=self.p2,
+                       threshold=w.threshold, min_commit=1, workspace=self.unmask_ws)
+        if ev is not None:
+            ev[4].record()
+
+    LAUNCHES_PER_STEP = 6   # select, build, rope_pack, attn_fwd, unmask partial, unmask commit
+
+
+# ----------------------------------------------------------------------------- helpers
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed loop runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.15)
+        self.proc.terminate()
+        self.proc.wait()
+        sm, mx, reasons, n = [], [], set(), 0
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                n += 1
+                for name, val in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"),
+                                     parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": n}
+
+
+def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        inp.step()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    if dist_on:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(steps):
+        inp.step(evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist_on:
+        torch.distributed.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    stages = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])  # ms
+    return total_ms, stages.mean(axis=0)
+
+
+def time_e2e(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
+    """The same step through the public API with host buffers: per step, the step's
+    inputs are copied from pinned host memory and the decode result is read back."""
+    ins = [inp.block_tokens, inp.topk_ids, inp.topk_prob, inp.q, inp.k, inp.v, inp.logits]
+    host_in = [t.cpu().pin_memory() for t in ins]
+    outs = [inp.commit, inp.argmax, inp.conf]
+    host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+
+    def one():
+        for d, h in zip(ins, host_in):
+            d.copy_(h, non_blocking=True)
+        inp.step()
+        for h, d in zip(host_out, outs):
+            h.copy_(d, non_blocking=True)
+
+    for _ in range(warmup):
+        one()
+    torch.cuda.synchronize()
+    if dist_on:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    torch.cuda.synchronize()
+    if dist_on:
+        torch.distributed.barrier()
+    return (time.perf_counter() - t0) * 1e3, h2d, d2h
+
+
+# ----------------------------------------------------------------------------- oracle arm
+
+
+class _RowView:
+    """Row access to a bf16 table as float64 without converting the whole table."""
+
+    def __init__(self, t: torch.Tensor):
+        self.t = t
+        self.shape = tuple(t.shape)
+
+    def __getitem__(self, i):
+        return self.t[int(i)].to(torch.float64).numpy()
+
+
+def oracle_sample(w: W.Workload, budget_s: float, seed: int = 99):
+    """Times the CPU oracle on whole denoising steps (selector, sparse input, attention,
+    unmasking) of the workload, block indices spread over the sweep, until `budget_s`
+    seconds of CPU work are spent.  Returns (steps/s, steps done, seconds, block indices)."""
+    from oracle import ssm_oracle as O
+    g = torch.Generator().manual_seed(seed)
+    V, H = w.vocab, w.hidden
+    embed = (torch.randn((V, H), generator=g)).to(torch.bfloat16)
+    ev = _RowView(embed)
+    mask_id = V - 1
+    order = list(w.block_indices)
+    if len(order) > 1:
+        # spread the sample over the sweep: 0, n/2, n/4, 3n/4, ...
+        spread, step = [], len(order)
+        seen = set()
+        while step >= 1:
+            for i in range(0, len(order), step):
+                if i not in seen:
+                    seen.add(i)
+                    spread.append(order[i])
+            step //= 2
+        order = spread
+    done, t_used, used = 0, 0.0, []
+    n_prefix = 0 if w.prefix_cached else w.prompt
+    for b in order * max(1, w.batch):
+        r, *_ = O.select_suffix(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
+        R = len(r)
+        n_new = n_prefix + w.block + R
+        n_cache = (w.prompt + b * w.block) if w.prefix_cached else 0
+        blk = torch.full((1, w.block), mask_id, dtype=torch.int32)
+        ids = torch.randint(0, V - 1, (1, R, w.topk), generator=g)
+        probs = torch.softmax(torch.randn((1, R, w.topk), generator=g) * 3, -1).double() * 0.5
+        pre = torch.randint(0, V - 1, (1, n_prefix), generator=g) if n_prefix else None
+        q = torch.randn((1, n_new, w.h_q, w.head_dim), generator=g).to(torch.bfloat16).double().numpy()
+        k = torch.randn((1, n_new, w.h_kv, w.head_dim), generator=g).to(torch.bfloat16).double().numpy()
+        v = torch.randn((1, n_new, w.h_kv, w.head_dim), generator=g).to(torch.bfloat16).double().numpy()
+        kc = torch.randn((1, n_cache, w.h_kv, w.head_dim), generator=g).to(torch.bfloat16).double().numpy()
+        vc = torch.randn((1, n_cache, w.h_kv, w.head_dim), generator=g).to(torch.bfloat16).double().numpy()
+        logits = (torch.randn((1, w.block, V), generator=g) * w.logits_sigma).to(torch.bfloat16).double().numpy()
+        masked = np.ones((1, w.block), dtype=np.uint8)
+        t0 = time.perf_counter()
+        r2, *_ = O.select_suffix(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
+        x, pos = O.build_step_input(ev, mask_id, blk.numpy(), W.block_start(w, b), r2, ids.numpy(), probs.numpy(),
+                                    w.alpha, prefix_tokens=None if pre is None else pre.numpy())
+        O.attention(q, k, v, pos, kc if n_cache else None, vc if n_cache else None, w.rope_theta)
+        O.unmask(logits, masked, O.MODE_THRESHOLD, w.threshold)
+        t_used += time.perf_counter() - t0
+        done += 1
+        used.append(b)
+        if t_used >= budget_s:
+            break
+    return done / t_used, done, t_used, used
+
+
+def reduce_max(x: float, device, dist_on: bool) -> float:
+    """Max over ranks of a per-rank time (the job ends when its slowest replica ends)."""
+    if not dist_on:
+        return float(x)
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, w: W.Workload, rank: int):
+    if rank != 0:
+        return
+    budget = max(1.0, float(os.environ.get("SSM_ORACLE_STEP_BUDGET_S", "8")))
+    rates = []
+    for _ in range(args.warmup):
+        oracle_sample(w, min(budget, 2.0))
+    t_total = 0.0
+    done_total = 0
+    for _ in range(args.steps):
+        rate, done, t, used = oracle_sample(w, budget)
+        rates.append(rate)
+        t_total += t
+        done_total += done
+    value = done_total / t_total
+    sample = (f"per bench step: whole denoising steps of the '{w.name}' workload on block indices spread over "
+              f"the sweep until {budget:.0f} s of CPU work; {done_total} denoising steps in {t_total:.1f} s")
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * t_total / max(args.steps, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": workload_desc(w), "parallelism": "replicas"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_desc(w: W.Workload) -> str:
+    blocks = (f"block indices {w.block_indices[0]}..{w.block_indices[-1]} as one batch"
+              if len(w.block_indices) > 1 else f"block index {w.block_indices[0]}")
+    cache = "prompt in a prefix KV cache" if w.prefix_cached else "prompt recomputed (no cache)"
+    return (f"{w.name}: {w.h_q}/{w.h_kv} heads, head_dim {w.head_dim}, hidden {w.hidden}, prompt {w.prompt} "
+            f"({cache}), gen {w.gen}, block {w.block}, budgets local {w.local}/middle {w.middle}/tail {w.tail}, "
+            f"batch {w.batch}, {blocks}, vocab {w.vocab} {w.logits_dtype} logits, top-k {w.topk}, alpha {w.alpha}, "
+            f"threshold {w.threshold}")
+
+
+# ----------------------------------------------------------------------------- main
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ssm", "reference"], default="ssm")
+    ap.add_argument("--workload", default="long", choices=list(W.WORKLOADS))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    w = W.WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, w, rank)
+        return
+
+    dist_on = world > 1
+    torch.cuda.set_device(local_rank)
+    if dist_on:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    from paper_2608_23167_gb300 import build_lib, ssm
+    if rank == 0 or not dist_on:
+        build_lib.build()
+    if dist_on:
+        torch.distributed.barrier()
+    ssm.lib()
+    dev = torch.device("cuda", local_rank)
+    inp = StepInputs(w, dev)
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    total_ms, stage_ms = time_steps(inp, args.steps, args.warmup, dist_on)
+    clk = clocks.stop()
+    err = ssm.ssm_get_device_error()
+    if err != 0:
+        raise RuntimeError(f"device error {err} during the timed region")
+
+    total_ms = reduce_max(total_ms, dev, dist_on)
+    units = inp.n * args.steps * world                 # denoising steps processed by all ranks
+    value = units / (total_ms / 1e3)
+
+    e2e = None
+    if not args.no_e2e:
+        e_ms, h2d, d2h = time_e2e(inp, args.steps, min(args.warmup, 5), dist_on)
+        e_ms = reduce_max(e_ms, dev, dist_on)
+        e2e = {"value": inp.n * args.steps * world / (e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+    peaks, peak_src = load_peaks()
+    sel_ms, build_ms, attn_ms, unmask_ms = [float(x) for x in stage_ms]
+    flops = inp.attn_flops()
+    attn_tflops = flops / (attn_ms * 1e-3) / 1e12
+    tensor_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+    hbm_peak = peaks["hbm_gbs"]
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", f"attention_{w.name}_traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            tr = json.load(f)
+        if tr.get("source_digest") == build_lib.source_digest("attention.cu"):
+            traffic = tr.get("dram_bytes_per_launch")
+    roofline = {"bound": "tensor", "achieved": attn_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
+                "frac": attn_tflops / tensor_peak, "traffic": traffic,
+                "kernel": "ssm_attention_varlen (rope_pack_kernel + attn_fwd_kernel)",
+                "peak_kind": f"bf16 dense, sustained ({peak_src})",
+                "algorithmic": f"{flops / 1e9:.1f} GFLOP per launch = 4 * heads * head_dim * sum(Nq * Nk)"}
+    gb = lambda nbytes, ms: nbytes / (ms * 1e-3) / 1e9  # noqa: E731
+    stages = {
+        "select_ms": sel_ms,
+        "build_ms": build_ms, "build_GBps": gb(inp.gather_bytes(), build_ms),
+        "build_frac_hbm": gb(inp.gather_bytes(), build_ms) / hbm_peak,
+        "attention_ms": attn_ms, "attention_TFLOPs": attn_tflops,
+        "attention_frac_bf16_sustained": attn_tflops / tensor_peak,
+        "attention_frac_bf16_burst": attn_tflops / peaks["bf16_tflops"],
+        "unmask_ms": unmask_ms, "unmask_GBps": gb(inp.unmask_bytes(), unmask_ms),
+        "unmask_frac_hbm": gb(inp.unmask_bytes(), unmask_ms) / hbm_peak,
+        "unmask_frac_8TBps_nominal": gb(inp.unmask_bytes(), unmask_ms) / 8000.0,
+    }
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        budget = float(os.environ.get("SSM_CPU_BASELINE_BUDGET_S", "15"))
+        rate, done, t_used, used = oracle_sample(w, budget)
+        cpu = {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+               "sample": f"{done} whole denoising steps (block indices {used}) of the same workload, "
+                         f"{t_used:.1f} s of CPU work, numpy fp64 with its default BLAS threads"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": workload_desc(w), "denoise_steps_per_bench_step": inp.n,
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "l2": "inputs larger than L2 (each step reads ~%.0f MB)" % (
+                           (inp.gather_bytes() + inp.attn_bytes() + inp.unmask_bytes()) / 1e6)},
+            "roofline": roofline, "stages": stages, "clocks": clk, "e2e": e2e,
+            "cpu_baseline": cpu, "gpu_launches": StepInputs.LAUNCHES_PER_STEP * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    if dist_on:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

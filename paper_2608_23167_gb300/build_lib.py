@@ -46,6 +46,12 @@ def _digest() -> str:
     return h.hexdigest()
 
 
+def source_digest(name: str) -> str:
+    """sha256 of one kernel source file (ties recorded profiler counters to a kernel version)."""
+    with open(os.path.join(CSRC, name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     """Compile (if sources changed) and return the path of libssm.so."""
     os.makedirs(BUILD, exist_ok=True)
