@@ -262,6 +262,31 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
                       int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
                       uint8_t* commit, void* workspace, size_t ws_bytes, ssm_stream_t stream);
 
+/* ssm_unmask_noalloc -- ssm_unmask for callers that cannot allocate device
+ * memory.  The paper has no counterpart: this is a deployment convenience.
+ *
+ * Some callers cannot call cudaMalloc or hand out a scratch buffer: a host
+ * program whose device memory is owned by another framework's allocator, or a
+ * code path where allocation is not permitted.  This entry point takes the
+ * same arguments as ssm_unmask minus the workspace and allocates nothing: its
+ * scratch is a fixed 1 MiB array in device global memory that the library
+ * holds on every GPU that loads it, until the process exits.
+ *   - Limit: ssm_unmask_workspace_size(batch, block_len, vocab, dtype) must be
+ *     at most 1 MiB (for example batch * block_len <= 4096 positions with a
+ *     126464-entry bf16 vocabulary); larger calls return SSM_ERR_CAPACITY and
+ *     enqueue nothing.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - Every call shares the one array: two calls that overlap on the GPU (on
+ *     different streams, or from different threads) race and corrupt each
+ *     other's results.  Serialise them.  The array keeps the last call's
+ *     contents; nothing in it needs to start at zero.
+ *   - No cudaMalloc, cudaFree or allocating library routine is called. */
+ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len,
+                              int64_t vocab, const uint8_t* masked, ssm_commit_mode mode, float threshold,
+                              int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
+                              uint8_t* commit, ssm_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -11,6 +11,8 @@
 // read.
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace ssm {
@@ -309,3 +311,55 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// ssm_unmask_noalloc: the same two kernels with their scratch in a fixed,
+// statically allocated device array instead of a caller workspace.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+// 1 MiB holds 65536 chunk partials: e.g. 128 sequences x 32 positions x 16
+// chunks of a 126464-entry bf16 vocabulary.  Every GPU that loads libssm
+// keeps this array until the process exits.
+constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;
+static __device__ __align__(256) unsigned char g_unmask_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_unmask_scratch on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up once
+// per device (with that device current) and cached.
+ssm_status scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return SSM_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_unmask_scratch) != cudaSuccess || p == nullptr) return SSM_ERR_CUDA;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return SSM_OK;
+}
+
+}  // namespace
+
+extern "C" ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len,
+                                         int64_t vocab, const uint8_t* masked, ssm_commit_mode mode,
+                                         float threshold, int32_t topk, int32_t min_commit, float* conf,
+                                         int32_t* argmax, float* p2, uint8_t* commit, ssm_stream_t stream) {
+  if (batch > 0 && block_len > 0 && vocab > 0 &&
+      ssm_unmask_workspace_size(batch, block_len, vocab, dtype) > kNoAllocScratchBytes)
+    return SSM_ERR_CAPACITY;
+  void* scratch = nullptr;
+  const ssm_status s = scratch_address(&scratch);
+  if (s != SSM_OK) return s;
+  // The chunk partials are written before they are read on every call, so the
+  // previous call's contents never need clearing.
+  return ssm_unmask(logits, dtype, batch, block_len, vocab, masked, mode, threshold, topk, min_commit, conf,
+                    argmax, p2, commit, scratch, kNoAllocScratchBytes, stream);
+}

@@ -78,6 +78,8 @@ def lib() -> ctypes.CDLL:
             "ssm_unmask_workspace_size": (sz, [i32, i32, i64, ctypes.c_int]),
             "ssm_unmask": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32, i32,
                                           vp, vp, vp, vp, vp, sz, vp]),
+            "ssm_unmask_noalloc": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32,
+                                                  i32, vp, vp, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -91,7 +93,7 @@ def exported_symbols() -> Sequence[str]:
     return ["ssm_status_str", "ssm_version", "ssm_get_device_error", "ssm_set_wait_limit_ns",
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
-            "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask"]
+            "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -276,3 +278,13 @@ def ssm_unmask(logits, masked, conf, argmax, commit, p2=None, mode: int = SSM_CO
         _ptr(logits), _dtype_code(logits), batch, block_len, vocab, _ptr(masked), mode, float(threshold), topk,
         min_commit, _ptr(conf), _ptr(argmax), _ptr(p2), _ptr(commit), _ptr(workspace), workspace.numel(),
         _stream(stream)))
+
+
+def ssm_unmask_noalloc(logits, masked, conf, argmax, commit, p2=None, mode: int = SSM_COMMIT_THRESHOLD,
+                       threshold: float = 0.9, topk: int = 1, min_commit: int = 1, stream=None):
+    """ssm_unmask without a workspace: for callers that cannot allocate device memory
+    (the library's fixed scratch array is used; concurrent calls race)."""
+    batch, block_len, vocab = logits.shape
+    _check("ssm_unmask_noalloc", lib().ssm_unmask_noalloc(
+        _ptr(logits), _dtype_code(logits), batch, block_len, vocab, _ptr(masked), mode, float(threshold), topk,
+        min_commit, _ptr(conf), _ptr(argmax), _ptr(p2), _ptr(commit), _stream(stream)))
