@@ -114,68 +114,83 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // RoPE + GQA packing of the new rows
 // ---------------------------------------------------------------------------
 
+constexpr int kRopeWarps = 8;
+
+// One warp per new row.  Each lane owns four rotation pairs (i, i + D/2) of one
+// head vector, so D/8 lanes cover a head and a warp moves 32/(D/8) heads per
+// pass with 8-byte loads and stores.  The angles pos * theta^(-2i/D) are formed
+// and reduced modulo 2*pi in fp64 (inverse frequencies once per CTA), then
+// sin/cos are taken in fp32 on the reduced angle.
 template <int D>
-__global__ void __launch_bounds__(128) rope_pack_kernel(
+__global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
-    const int32_t* __restrict__ pos, AttnParams p, float theta, __nv_bfloat16* __restrict__ qhat,
-    __nv_bfloat16* __restrict__ khat) {
-  constexpr int PPL = D / 64;  // rotation pairs per lane
+    const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max,
+    __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
+  constexpr int LPH = D / 8;        // lanes per head vector
+  constexpr int HPP = 32 / LPH;     // head vectors per warp pass
+  __shared__ double inv_freq[D / 2];
+  if (threadIdx.x < D / 2)
+    inv_freq[threadIdx.x] = theta > 0.f ? exp2(-(2.0 * threadIdx.x / D) * log2(static_cast<double>(theta))) : 0.0;
+  __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int sub = lane % LPH;       // which 4 pairs
+  const int hoff = lane / LPH;      // which head of the pass
   const int prob = blockIdx.y;
   const Geom gm = problem_geom(p, prob);
-  const int i = blockIdx.x * 4 + warp;
+  const int i = blockIdx.x * kRopeWarps + warp;
   if (i >= gm.n_new) return;
   const int32_t ps = pos[p.problems ? gm.new_row + i : i];
-  float cs[PPL], sn[PPL];
+  float cs[4], sn[4];
 #pragma unroll
-  for (int t = 0; t < PPL; ++t) {
-    if (theta > 0.f) {
-      const int jp = lane * PPL + t;
-      const double inv = pow(static_cast<double>(theta), -2.0 * jp / D);
-      double s, c;
-      sincos(static_cast<double>(ps) * inv, &s, &c);
-      cs[t] = static_cast<float>(c);
-      sn[t] = static_cast<float>(s);
-    } else {
-      cs[t] = 1.f;
-      sn[t] = 0.f;
-    }
+  for (int t = 0; t < 4; ++t) {
+    const double a = static_cast<double>(ps) * inv_freq[4 * sub + t];
+    const double kk = rint(a * 0.15915494309189535);               // a / (2 pi)
+    double r = fma(-kk, 6.283185307179586, a);                      // 2 pi, high part
+    r = fma(-kk, 2.4492935982947064e-16, r);                        // 2 pi, low part
+    sincosf(static_cast<float>(r), &sn[t], &cs[t]);
   }
-  auto rotate = [&](const __nv_bfloat16* src, __nv_bfloat16* dst) {
-    float x1[PPL], x2[PPL];
-    if constexpr (PPL == 2) {
-      const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(src + 2 * lane);
-      const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(src + D / 2 + 2 * lane);
-      x1[0] = __low2float(a);
-      x1[1] = __high2float(a);
-      x2[0] = __low2float(b);
-      x2[1] = __high2float(b);
-    } else {
-      x1[0] = __bfloat162float(src[lane]);
-      x2[0] = __bfloat162float(src[D / 2 + lane]);
-    }
-    float y1[PPL], y2[PPL];
-#pragma unroll
-    for (int t = 0; t < PPL; ++t) {
-      y1[t] = x1[t] * cs[t] - x2[t] * sn[t];
-      y2[t] = x2[t] * cs[t] + x1[t] * sn[t];
-    }
-    if constexpr (PPL == 2) {
-      *reinterpret_cast<__nv_bfloat162*>(dst + 2 * lane) = __floats2bfloat162_rn(y1[0], y1[1]);
-      *reinterpret_cast<__nv_bfloat162*>(dst + D / 2 + 2 * lane) = __floats2bfloat162_rn(y2[0], y2[1]);
-    } else {
-      dst[lane] = __float2bfloat16_rn(y1[0]);
-      dst[D / 2 + lane] = __float2bfloat16_rn(y2[0]);
-    }
-  };
   const int64_t row = gm.new_row + i;
-  for (int h = 0; h < p.h_q; ++h) {
-    const int g = h / p.grp, hl = h - g * p.grp;
-    const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
-                            static_cast<int64_t>(i) * p.grp + hl;
-    rotate(q + (row * p.h_q + h) * D, qhat + dst_row * D);
+  const int n_vec = p.h_q + p.h_kv;
+  for (int base = 0; base < n_vec; base += HPP * 4) {
+    uint2 x1[4], x2[4];
+    int hv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      hv[u] = base + u * HPP + hoff;
+      if (hv[u] < n_vec) {
+        const __nv_bfloat16* src = hv[u] < p.h_q ? q + (row * p.h_q + hv[u]) * D
+                                                 : k + (row * p.h_kv + (hv[u] - p.h_q)) * D;
+        x1[u] = *reinterpret_cast<const uint2*>(src + 4 * sub);
+        x2[u] = *reinterpret_cast<const uint2*>(src + D / 2 + 4 * sub);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (hv[u] >= n_vec) continue;
+      const float a[4] = {__uint_as_float(x1[u].x << 16), __uint_as_float(x1[u].x & 0xFFFF0000u),
+                          __uint_as_float(x1[u].y << 16), __uint_as_float(x1[u].y & 0xFFFF0000u)};
+      const float b[4] = {__uint_as_float(x2[u].x << 16), __uint_as_float(x2[u].x & 0xFFFF0000u),
+                          __uint_as_float(x2[u].y << 16), __uint_as_float(x2[u].y & 0xFFFF0000u)};
+      float y1[4], y2[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        y1[t] = a[t] * cs[t] - b[t] * sn[t];
+        y2[t] = b[t] * cs[t] + a[t] * sn[t];
+      }
+      __nv_bfloat16* dst;
+      if (hv[u] < p.h_q) {
+        const int g = hv[u] / p.grp, hl = hv[u] - g * p.grp;
+        const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
+                                static_cast<int64_t>(i) * p.grp + hl;
+        dst = qhat + dst_row * D;
+      } else {
+        dst = khat + (row * p.h_kv + (hv[u] - p.h_q)) * D;
+      }
+      *reinterpret_cast<uint2*>(dst + 4 * sub) = make_uint2(pack_bf16x2(y1[0], y1[1]), pack_bf16x2(y1[2], y1[3]));
+      *reinterpret_cast<uint2*>(dst + D / 2 + 4 * sub) =
+          make_uint2(pack_bf16x2(y2[0], y2[1]), pack_bf16x2(y2[2], y2[3]));
+    }
   }
-  for (int g = 0; g < p.h_kv; ++g) rotate(k + (row * p.h_kv + g) * D, khat + (row * p.h_kv + g) * D);
 }
 
 // ---------------------------------------------------------------------------
@@ -566,10 +581,10 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.wait_ns = wait_limit_ns();
   const int n_prob = batch_or_np;
   {
-    dim3 grid((max_n_new + 3) / 4, n_prob);
-    rope_pack_kernel<D><<<grid, 128, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
-                                               static_cast<const __nv_bfloat16*>(k_new), pos, p, rope_theta,
-                                               qhat, khat);
+    dim3 grid((max_n_new + kRopeWarps - 1) / kRopeWarps, n_prob);
+    rope_pack_kernel<D><<<grid, kRopeWarps * 32, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
+                                                          static_cast<const __nv_bfloat16*>(k_new), pos, p,
+                                                          rope_theta, max_n_new, qhat, khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK) return s;
   }

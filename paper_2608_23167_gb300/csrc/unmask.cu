@@ -19,7 +19,7 @@ namespace ssm {
 namespace {
 
 constexpr int kUnmaskThreads = 256;
-constexpr int kUnroll = 4;                         // 16-byte vectors per thread per chunk
+constexpr int kUnroll = 16;                        // 16-byte vectors per thread per chunk
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Partial {
@@ -102,10 +102,110 @@ struct Vec<float> {
   __device__ static float scalar(const float* p, int64_t i) { return p[i]; }
 };
 
-// Chunk of `chunk` elements (a multiple of kUnmaskThreads * kUnroll * VEC when
-// VECTOR) of row blockIdx.y.
-template <typename T, bool VECTOR>
-__global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_kernel(
+// Block-wide reductions over the 256 threads of a CTA (result in every thread).
+__device__ __forceinline__ float block_max(float v, float* red) {
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, d));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  v = red[lane & (kUnmaskThreads / 32 - 1)];
+#pragma unroll
+  for (int d = kUnmaskThreads / 64; d >= 1; d >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, d));
+  return v;
+}
+
+// Chunk of one row: thread t holds vectors t, t + 256, ..., t + 256 (U - 1) of
+// the chunk (16 bytes each, so a warp reads 512 contiguous bytes per vector).
+// Pass 1 keeps the two largest values per thread; after the block maximum M is
+// known, pass 2 sums exp(x - M) and the holder(s) of M report its first index.
+template <typename T, int U>
+__global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_vec_kernel(
+    const T* __restrict__ logits, int64_t vocab, int64_t chunk, int n_chunks,
+    const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
+  constexpr int N = Vec<T>::N;
+  __shared__ float red_f[kUnmaskThreads / 32];
+  __shared__ Partial red_p[kUnmaskThreads / 32];
+  const int64_t row = blockIdx.y;
+  if (!masked[row]) return;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * chunk;
+  const int64_t c1 = min(vocab, c0 + chunk);
+  const uint4* xv = reinterpret_cast<const uint4*>(logits + row * vocab);
+  uint4 v[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
+    v[u] = (e < c1) ? __ldcs(xv + e / N) : make_uint4(0, 0, 0, 0);
+  }
+  float m1 = -INFINITY, m2 = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
+    if (e < c1) {
+      float f[N];
+      Vec<T>::unpack(v[u], f);
+#pragma unroll
+      for (int c = 0; c < N; ++c) {
+        m2 = fmaxf(m2, fminf(m1, f[c]));
+        m1 = fmaxf(m1, f[c]);
+      }
+    }
+  }
+  const float M = block_max(m1, red_f);
+  const float mb = (M == -INFINITY) ? 0.f : M * kLog2e;  // a chunk of -inf logits sums to 0
+  float s = 0.f;
+  int idx = INT_MAX;
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
+    if (e < c1) {
+      float f[N];
+      Vec<T>::unpack(v[u], f);
+#pragma unroll
+      for (int c = 0; c < N; ++c) s += ex2(fmaf(f[c], kLog2e, -mb));
+      if (m1 == M && idx == INT_MAX) {
+#pragma unroll
+        for (int c = 0; c < N; ++c)
+          if (f[c] == M && idx == INT_MAX) idx = static_cast<int>(e + c);
+      }
+    }
+  }
+  // (m, s, idx, second): a thread whose maximum is below M offers it as a second
+  // candidate; two threads holding M make M itself the second-largest value.
+  Partial p{M, s, idx, (m1 == M) ? m2 : m1};
+  int holders = (m1 == M) ? 1 : 0;
+#pragma unroll
+  for (int d = 16; d >= 1; d >>= 1) {
+    p.s += __shfl_xor_sync(0xffffffffu, p.s, d);
+    p.idx = min(p.idx, __shfl_xor_sync(0xffffffffu, p.idx, d));
+    p.m2 = fmaxf(p.m2, __shfl_xor_sync(0xffffffffu, p.m2, d));
+    holders += __shfl_xor_sync(0xffffffffu, holders, d);
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    p.m = __int_as_float(holders);  // the warp's holder count rides in the unused m field
+    red_p[warp] = p;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    Partial q = red_p[lane & (kUnmaskThreads / 32 - 1)];
+    int h = (lane < kUnmaskThreads / 32) ? __float_as_int(q.m) : 0;
+    if (lane >= kUnmaskThreads / 32) q = Partial{0.f, 0.f, INT_MAX, -INFINITY};
+#pragma unroll
+    for (int d = kUnmaskThreads / 64; d >= 1; d >>= 1) {
+      q.s += __shfl_xor_sync(0xffffffffu, q.s, d);
+      q.idx = min(q.idx, __shfl_xor_sync(0xffffffffu, q.idx, d));
+      q.m2 = fmaxf(q.m2, __shfl_xor_sync(0xffffffffu, q.m2, d));
+      h += __shfl_xor_sync(0xffffffffu, h, d);
+    }
+    if (lane == 0) part[row * n_chunks + blockIdx.x] = Partial{M, q.s, q.idx, (h >= 2) ? M : q.m2};
+  }
+}
+
+// Rows whose length or alignment rules out 16-byte vectors: one element per
+// thread per step, online (max, second, first index) then the exp sum.
+template <typename T>
+__global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_scalar_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t chunk, int n_chunks,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
   const int64_t row = blockIdx.y;
@@ -116,41 +216,12 @@ __global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_kernel(
   float m = -INFINITY, m2 = -INFINITY;
   int idx = INT_MAX;
   float s = 0.f;
-  if constexpr (VECTOR) {
-    constexpr int N = Vec<T>::N;
-    uint4 v[kUnroll];
-    const uint4* xv = reinterpret_cast<const uint4*>(x);
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
-      v[u] = (e < c1) ? __ldcs(xv + e / N) : make_uint4(0, 0, 0, 0);
-    }
-    float f[kUnroll][N];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      Vec<T>::unpack(v[u], f[u]);
-      const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
-#pragma unroll
-      for (int c = 0; c < N; ++c) {
-        if (e + c < c1) observe(f[u][c], static_cast<int>(e + c), m, idx, m2);
-        else f[u][c] = -INFINITY;
-      }
-    }
-    if (m > -INFINITY) {
-      const float mb = m * kLog2e;
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u)
-#pragma unroll
-        for (int c = 0; c < N; ++c) s += ex2(fmaf(f[u][c], kLog2e, -mb));
-    }
-  } else {
+  for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
+    observe(Vec<T>::scalar(x, e), static_cast<int>(e), m, idx, m2);
+  if (m > -INFINITY) {
+    const float mb = m * kLog2e;
     for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
-      observe(Vec<T>::scalar(x, e), static_cast<int>(e), m, idx, m2);
-    if (m > -INFINITY) {
-      const float mb = m * kLog2e;
-      for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
-        s += ex2(fmaf(Vec<T>::scalar(x, e), kLog2e, -mb));
-    }
+      s += ex2(fmaf(Vec<T>::scalar(x, e), kLog2e, -mb));
   }
   Partial p{m, s, idx, m2};
 #pragma unroll
@@ -242,8 +313,8 @@ UnmaskPlan plan_unmask(int64_t vocab, ssm_dtype dtype, const void* logits) {
   const int vec = 16 / esz;
   UnmaskPlan p;
   p.vector = ((vocab * esz) % 16 == 0) && (logits == nullptr || ssm::aligned16(logits));
-  p.chunk = p.vector ? static_cast<int64_t>(ssm::kUnmaskThreads) * ssm::kUnroll * vec
-                     : static_cast<int64_t>(ssm::kUnmaskThreads) * 16;
+  // both plans cut a row into the same chunks, so the workspace does not depend on the plan
+  p.chunk = static_cast<int64_t>(ssm::kUnmaskThreads) * ssm::kUnroll * vec;
   p.n_chunks = static_cast<int>((vocab + p.chunk - 1) / p.chunk);
   return p;
 }
@@ -254,11 +325,8 @@ extern "C" {
 
 size_t ssm_unmask_workspace_size(int32_t batch, int32_t block_len, int64_t vocab, ssm_dtype dtype) {
   if (batch <= 0 || block_len <= 0 || vocab <= 0) return 0;
-  // the scalar plan has the most chunks; size for it so either plan fits
-  const int64_t n_chunks = (vocab + ssm::kUnmaskThreads * 16 - 1) / (ssm::kUnmaskThreads * 16);
-  const UnmaskPlan v = plan_unmask(vocab, dtype, nullptr);
-  const int64_t nc = n_chunks > v.n_chunks ? n_chunks : v.n_chunks;
-  return ssm::align_up(static_cast<size_t>(batch) * block_len * nc * sizeof(ssm::Partial), 256);
+  const UnmaskPlan plan = plan_unmask(vocab, dtype, nullptr);
+  return ssm::align_up(static_cast<size_t>(batch) * block_len * plan.n_chunks * sizeof(ssm::Partial), 256);
 }
 
 ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len,
@@ -286,18 +354,18 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
     if (plan.vector)
-      ssm::unmask_partial_kernel<__nv_bfloat16, true><<<grid, ssm::kUnmaskThreads, 0, st>>>(
+      ssm::unmask_partial_vec_kernel<__nv_bfloat16, ssm::kUnroll><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
     else
-      ssm::unmask_partial_kernel<__nv_bfloat16, false><<<grid, ssm::kUnmaskThreads, 0, st>>>(
+      ssm::unmask_partial_scalar_kernel<__nv_bfloat16><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
   } else {
     auto* x = static_cast<const float*>(logits);
     if (plan.vector)
-      ssm::unmask_partial_kernel<float, true><<<grid, ssm::kUnmaskThreads, 0, st>>>(
+      ssm::unmask_partial_vec_kernel<float, ssm::kUnroll><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
     else
-      ssm::unmask_partial_kernel<float, false><<<grid, ssm::kUnmaskThreads, 0, st>>>(
+      ssm::unmask_partial_scalar_kernel<float><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
   }
   ssm_status s = ssm::launch_status();
@@ -319,7 +387,7 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
 
 namespace {
 
-// 1 MiB holds 65536 chunk partials: e.g. 128 sequences x 32 positions x 16
+// 1 MiB holds 65536 chunk partials: e.g. 512 sequences x 32 positions x 4
 // chunks of a 126464-entry bf16 vocabulary.  Every GPU that loads libssm
 // keeps this array until the process exits.
 constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;

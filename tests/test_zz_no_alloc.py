@@ -56,6 +56,7 @@ def test_unmask_noalloc_rejects_sizes_beyond_its_scratch():
     build_lib.build()
     lib = ssm.lib()
     fake = 1 << 20
-    # 2048 rows x 16 chunks x 16 bytes = 512 KiB fits; 8192 rows x 16 chunks = 2 MiB does not
-    assert lib.ssm_unmask_noalloc(fake, 0, 256, 32, 126464, fake, 0, ctypes.c_float(0.9), 1, 1, fake, fake,
+    # 126464-entry bf16 rows are 4 chunks of 16-byte partials: 16384 positions fill 1 MiB exactly
+    assert lib.ssm_unmask_workspace_size(512, 32, 126464, 0) == 1 << 20
+    assert lib.ssm_unmask_noalloc(fake, 0, 513, 32, 126464, fake, 0, ctypes.c_float(0.9), 1, 1, fake, fake,
                                   fake, fake, None) == 3
