@@ -5,19 +5,21 @@
 //
 // Two kernels:
 //  * rope_pack_kernel rotates the new queries and keys at their original
-//    positions (fp64 angles, fp32 rotation, bf16 store) and packs the queries
-//    of one GQA group into one row block, (query i, head-in-group hl) -> row
-//    i * grp + hl, so that a 128-row M tile of the tensor-core GEMM is filled
-//    with every query head that shares a key/value head.
-//  * attn_fwd_kernel: one CTA per (problem, kv head, 128-row query tile).
-//    Warp 0 streams K/V tiles with TMA (128 keys = four 32-row sub-boxes, so
-//    the cache segment and the new-row segment pack back to back with at most
-//    31 padded keys each); warp 1 issues tcgen05.mma (S = Q K^T and O += P V,
-//    bf16 operands from shared memory, fp32 accumulators in tensor memory);
-//    warps 2-5 run the online softmax, one query row per thread, reading S
-//    from tensor memory and writing P (bf16) to shared memory.  S is double
-//    buffered in tensor memory so QK^T of tile j+1 overlaps the softmax of
-//    tile j.  O is rescaled only when a row maximum grows by more than 2^8.
+//    positions and packs the queries of one GQA group into one row block,
+//    (query i, head-in-group hl) -> row i * grp + hl, so that a 128-row M tile
+//    of the tensor-core GEMM holds every query head that shares a K/V head.
+//  * attn_fwd_kernel: one CTA per (problem, kv head, pair of 128-row query
+//    tiles).  Warp 0 streams K/V tiles with TMA (128 keys = four 32-row
+//    sub-boxes, so the cache segment and the new-row segment pack back to back
+//    with at most 31 padded keys each; 3-stage K ring, 2-stage V ring).  Warp 1
+//    issues tcgen05.mma: S = Q K^T from shared memory into tensor memory, and
+//    O += P V with P read from tensor memory.  Two softmax warpgroups ("slots"
+//    A and B, one query row per thread) alternate: while one turns its S tile
+//    into P (written back over S as bf16), the tensor core runs the other
+//    slot's GEMMs.  With two query tiles each slot owns one; with a single
+//    query tile the slots split the key tiles (even/odd) and merge their
+//    partial softmax states at the end.  O is rescaled only when a row maximum
+//    grows by more than 2^8.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
@@ -34,40 +36,41 @@ namespace {
 constexpr int kBM = 128;            // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;            // keys per tile (tcgen05 N of QK^T, K of PV)
 constexpr int kSub = 32;            // rows per TMA sub-box of a key tile
-constexpr int kAttnThreads = 192;   // warp 0: TMA, warp 1: MMA, warps 2-5: softmax
+constexpr int kAttnThreads = 320;   // warp 0: TMA, warp 1: MMA, warps 2-5: slot A, warps 6-9: slot B
 constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
+constexpr int kKStages = 3;
+constexpr int kVStages = 2;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kOCol = 256;       // O accumulator columns; S buffers at 0 and 128
+constexpr uint32_t kOCol = 256;       // O of slot X at 256 + X * D; S (and P) of slot X at X * 128
 constexpr uint64_t kDrainNs = 200000000ull;
 
 enum Bar {
   Q_FULL = 0,
-  K_FULL = 1,   // [2]
-  K_EMPTY = 3,  // [2]
-  V_FULL = 5,   // [2]
-  V_EMPTY = 7,  // [2]
-  S_FULL = 9,   // [2]
-  S_FREE = 11,  // [2]
-  P_FULL = 13,  // [2]
-  P_FREE = 15,  // [2]
-  O_DONE = 17,
-  DRAIN = 18,
-  N_BARS = 19
+  K_FULL = 1,
+  K_EMPTY = K_FULL + kKStages,
+  V_FULL = K_EMPTY + kKStages,
+  V_EMPTY = V_FULL + kVStages,
+  S_FULL = V_EMPTY + kVStages,  // [2]: one per slot
+  P_FULL = S_FULL + 2,          // [2]
+  O_DONE = P_FULL + 2,          // [2]
+  DRAIN = O_DONE + 2,
+  N_BARS = DRAIN + 1
 };
 
 template <int D>
 struct Layout {
-  static constexpr int NP = D / 64;                 // 64-column panels per row
-  static constexpr int Q = 0;
-  static constexpr int K = Q + NP * kPanel;         // 2 stages
-  static constexpr int V = K + 2 * NP * kPanel;     // 2 stages
-  static constexpr int P = V + 2 * NP * kPanel;     // 2 buffers of 128 x 128 bf16
-  static constexpr int BAR = P + 2 * 2 * kPanel;
-  static constexpr int BYTES = BAR + N_BARS * 8 + 8;
-  static constexpr int ALLOC = BYTES + 1024;        // slack to align the base to 1024 B
+  static constexpr int NP = D / 64;                   // 64-column panels per row
+  static constexpr int TILE = NP * kPanel;            // one 128-row tile
+  static constexpr int Q = 0;                         // two query tiles
+  static constexpr int K = Q + 2 * TILE;
+  static constexpr int V = K + kKStages * TILE;
+  static constexpr int BAR = V + kVStages * TILE;
+  static constexpr int MERGE = BAR + N_BARS * 8 + 8;  // split-key merge: (m, l) per row
+  static constexpr int BYTES = MERGE + 2 * kBM * 4;
+  static constexpr int ALLOC = BYTES + 1024;          // slack to align the base to 1024 B
   static_assert(ALLOC <= 232448, "shared memory budget");
 };
 
@@ -197,6 +200,23 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
 // Attention forward
 // ---------------------------------------------------------------------------
 
+// Valid keys in each 32-row sub-box of key tile j (cache sub-boxes first, then
+// new-row sub-boxes); returns true if all 128 keys of the tile are valid.
+__device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub, const Geom& gm, int (&vcnt)[4]) {
+  bool full = true;
+#pragma unroll
+  for (int s4 = 0; s4 < 4; ++s4) {
+    const int sub = 4 * j + s4;
+    int c;
+    if (sub < n_csub) c = min(kSub, gm.n_cache - sub * kSub);
+    else if (sub - n_csub < n_nsub) c = min(kSub, gm.n_new - (sub - n_csub) * kSub);
+    else c = 0;
+    vcnt[s4] = c;
+    full = full && (c == kSub);
+  }
+  return full;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
@@ -211,32 +231,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + N_BARS);
+  float* merge_m = reinterpret_cast<float*>(smem + L::MERGE);
+  float* merge_l = merge_m + kBM;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int prob = blockIdx.y / p.h_kv;
   const int g = blockIdx.y - prob * p.h_kv;
-  const int mt = blockIdx.x;
   const Geom gm = problem_geom(p, prob);
   const int rows_q = gm.n_new * p.grp;
-  if (mt * kBM >= rows_q) return;  // whole CTA, before any shared state exists
+  const int n_qt = (rows_q + kBM - 1) / kBM;
+  const int qt0 = 2 * blockIdx.x;            // first query tile of this CTA
+  if (qt0 >= n_qt) return;                   // whole CTA, before any shared state exists
+  const bool two = qt0 + 1 < n_qt;           // two query tiles, else the slots split the keys
   const bool uniform = p.problems == nullptr;
   const int n_csub = (gm.n_cache + kSub - 1) / kSub;
   const int n_nsub = (gm.n_new + kSub - 1) / kSub;
-  const int nt = (n_csub + n_nsub + 3) / 4;
+  const int nt = (n_csub + n_nsub + 3) / 4;  // key tiles
+  const int n_jobs = two ? 2 * nt : nt;      // job t: slot t & 1, key tile two ? t >> 1 : t
 
   if (threadIdx.x == 0) {
     mbar_init(&bars[Q_FULL], 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       mbar_init(&bars[K_FULL + s], 1);
       mbar_init(&bars[K_EMPTY + s], 1);
+    }
+    for (int s = 0; s < kVStages; ++s) {
       mbar_init(&bars[V_FULL + s], 1);
       mbar_init(&bars[V_EMPTY + s], 1);
-      mbar_init(&bars[S_FULL + s], 1);
-      mbar_init(&bars[S_FREE + s], 128);
-      mbar_init(&bars[P_FULL + s], 128);
-      mbar_init(&bars[P_FREE + s], 1);
     }
-    mbar_init(&bars[O_DONE], 1);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&bars[S_FULL + x], 1);
+      mbar_init(&bars[P_FULL + x], 128);
+      mbar_init(&bars[O_DONE + x], 1);
+    }
     mbar_init(&bars[DRAIN], 1);
     fence_mbar_init();
   }
@@ -260,31 +287,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
-      int issued_k[2] = {0, 0}, issued_v[2] = {0, 0};
-      mbar_arrive_expect_tx(&bars[Q_FULL], NP * kPanel);
-      int qy, qz;
-      if (uniform) {
-        qy = mt * kBM;
-        qz = prob * p.h_kv + g;
-      } else {
-        qy = static_cast<int>((gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp) + mt * kBM;
-        qz = 0;
-      }
+      int last_k = -1, last_v = -1;  // latest K / V tile whose load was issued
+      const int nq = two ? 2 : 1;
+      mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
+      for (int x = 0; x < nq; ++x) {
+        int qy, qz;
+        if (uniform) {
+          qy = (qt0 + x) * kBM;
+          qz = prob * p.h_kv + g;
+        } else {
+          qy = static_cast<int>((gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp) + (qt0 + x) * kBM;
+          qz = 0;
+        }
 #pragma unroll
-      for (int pn = 0; pn < NP; ++pn) tma_load_3d(smem + L::Q + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+        for (int pn = 0; pn < NP; ++pn)
+          tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+      }
       const int c3 = uniform ? prob : 0;
-      for (int j = 0; j < nt && ok; ++j) {
-        const int st = j & 1;
-        const uint32_t empty_par = ((j >> 1) - 1) & 1;
-        for (int half = 0; half < 2 && ok; ++half) {  // half 0: K, half 1: V
-          if (j >= 2) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], empty_par, p.wait_ns);
+      // K runs one tile ahead of V: K(j) then V(j - 1)
+      for (int j = 0; j <= nt && ok; ++j) {
+        for (int half = 0; half < 2 && ok; ++half) {
+          const int jt = half ? j - 1 : j;
+          if (jt < 0 || jt >= nt) continue;
+          const int nst = half ? kVStages : kKStages;
+          const int st = jt % nst;
+          const int fill = jt / nst;
+          if (fill > 0) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
           if (!ok) break;
           uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
-          mbar_arrive_expect_tx(full, NP * kPanel);
-          uint8_t* dst = smem + (half ? L::V : L::K) + st * NP * kPanel;
+          mbar_arrive_expect_tx(full, L::TILE);
+          uint8_t* dst = smem + (half ? L::V : L::K) + st * L::TILE;
 #pragma unroll
           for (int sb = 0; sb < 4; ++sb) {
-            const int sub = 4 * j + sb;
+            const int sub = 4 * jt + sb;
             const CUtensorMap* map;
             int c2;
             if (sub < n_csub) {
@@ -301,18 +336,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
             for (int pn = 0; pn < NP; ++pn)
               tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, g, c2, c3);
           }
-          if (half) ++issued_v[st];
-          else ++issued_k[st];
+          if (half) last_v = jt;
+          else last_k = jt;
         }
       }
       if (!ok) {
         record_error(p.err, SSM_ERR_TIMEOUT);
-        // let every copy in flight land before the CTA's shared memory is released
+        // let every copy in flight land before the CTA's shared memory is released:
+        // the newest fill of each stage is the only one that can still be in flight
         mbar_wait(&bars[Q_FULL], 0, kDrainNs);
-        for (int s = 0; s < 2; ++s) {
-          if (issued_k[s]) mbar_wait(&bars[K_FULL + s], (issued_k[s] - 1) & 1, kDrainNs);
-          if (issued_v[s]) mbar_wait(&bars[V_FULL + s], (issued_v[s] - 1) & 1, kDrainNs);
-        }
+        for (int jt = max(0, last_k - kKStages + 1); jt <= last_k; ++jt)
+          mbar_wait(&bars[K_FULL + jt % kKStages], (jt / kKStages) & 1, kDrainNs);
+        for (int jt = max(0, last_v - kVStages + 1); jt <= last_v; ++jt)
+          mbar_wait(&bars[V_FULL + jt % kVStages], (jt / kVStages) & 1, kDrainNs);
       }
     }
     __syncwarp();
@@ -324,43 +360,51 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       const uint32_t sQ = smem_u32(smem + L::Q);
       const uint32_t sK = smem_u32(smem + L::K);
       const uint32_t sV = smem_u32(smem + L::V);
-      const uint32_t sP = smem_u32(smem + L::P);
-      for (int j = 0; j <= nt && ok; ++j) {
-        if (j < nt) {
-          const int sb = j & 1;
-          ok = mbar_wait(&bars[K_FULL + sb], (j >> 1) & 1, p.wait_ns);
-          if (ok && j >= 2) ok = mbar_wait(&bars[S_FREE + sb], ((j >> 1) - 1) & 1, p.wait_ns);
-          if (!ok) break;
-          tc_fence_after_sync();
-          const uint32_t kb = sK + sb * NP * kPanel;
+      int kx0 = 0, kx1 = 0;        // jobs issued per slot
+      int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
+      // O_X += P_X V(j) for slot X's latest job
+      auto issue_pv = [&](int x) -> bool {
+        const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
+        if (!mbar_wait(&bars[P_FULL + x], k & 1, p.wait_ns)) return false;
+        if (!mbar_wait(&bars[V_FULL + jp % kVStages], (jp / kVStages) & 1, p.wait_ns)) return false;
+        tc_fence_after_sync();
+        const uint32_t vb = sV + (jp % kVStages) * L::TILE;
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
-            umma_bf16_ss(tmem + sb * kBN, sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024),
-                         kIdescQK, kk > 0 ? 1u : 0u);
-          }
-          umma_commit(&bars[S_FULL + sb]);
-          umma_commit(&bars[K_EMPTY + sb]);
+        for (int kk = 0; kk < kBN / 16; ++kk)
+          umma_bf16_ts(tmem + kOCol + x * D, tmem + x * kBN + kk * 8, sdesc_sw128(vb + kk * 16 * 128, kPanel, 1024),
+                       kIdescPV, (k > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&bars[O_DONE + x]);
+        if (!two || x == 1) umma_commit(&bars[V_EMPTY + jp % kVStages]);
+        return true;
+      };
+      for (int t = 0; t < n_jobs && ok; ++t) {
+        const int x = t & 1;
+        const int j = two ? (t >> 1) : t;
+        if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
+        if (!ok) break;
+        ok = mbar_wait(&bars[K_FULL + j % kKStages], (j / kKStages) & 1, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after_sync();
+        const uint32_t qb = sQ + (two ? x : 0) * L::TILE;
+        const uint32_t kb = sK + (j % kKStages) * L::TILE;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
+          umma_bf16_ss(tmem + x * kBN, sdesc_sw128(qb + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024), kIdescQK,
+                       kk > 0 ? 1u : 0u);
         }
-        if (j >= 1) {
-          const int jj = j - 1, pb = jj & 1;
-          ok = mbar_wait(&bars[P_FULL + pb], (jj >> 1) & 1, p.wait_ns);
-          if (ok) ok = mbar_wait(&bars[V_FULL + pb], (jj >> 1) & 1, p.wait_ns);
-          if (!ok) break;
-          tc_fence_after_sync();
-          const uint32_t vb = sV + pb * NP * kPanel;
-          const uint32_t pbuf = sP + pb * 2 * kPanel;
-#pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk) {
-            const uint64_t ad = sdesc_sw128(pbuf + (kk >> 2) * kPanel + (kk & 3) * 32, 16, 1024);
-            const uint64_t bd = sdesc_sw128(vb + kk * 16 * 128, kPanel, 1024);
-            umma_bf16_ss(tmem + kOCol, ad, bd, kIdescPV, (jj > 0 || kk > 0) ? 1u : 0u);
-          }
-          umma_commit(&bars[O_DONE]);
-          umma_commit(&bars[V_EMPTY + pb]);
-          umma_commit(&bars[P_FREE + pb]);
+        umma_commit(&bars[S_FULL + x]);
+        if (!two || x == 1) umma_commit(&bars[K_EMPTY + j % kKStages]);
+        if (x) {
+          jlast1 = j;
+          ++kx1;
+        } else {
+          jlast0 = j;
+          ++kx0;
         }
       }
+      if (ok && kx0 > 0) ok = issue_pv(0);
+      if (ok && kx1 > 0) ok = issue_pv(1);
       if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
       // every issued MMA completes before tensor memory is released
       umma_commit(&bars[DRAIN]);
@@ -368,37 +412,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------- softmax (warps 2..5)
-    const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31 belong to this warp
+    // ------------------------------------------------------------- softmax slots (warps 2..9)
+    const int x = (warp - 2) >> 2;   // slot
+    const int quarter = warp & 3;    // TMEM lanes 32*quarter .. +31 belong to this warp
     const int row = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
-    const uint32_t sP = smem_u32(smem + L::P);
+    const uint32_t tS = tmem + lane_off + x * kBN;
+    const uint32_t tO = tmem + lane_off + kOCol + x * D;
+    const int jobs = two ? nt : (x == 0 ? (nt + 1) / 2 : nt / 2);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int j = 0; j < nt; ++j) {
-      const int sb = j & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[S_FULL + sb], (j >> 1) & 1, p.wait_ns));
+    for (int k = 0; k < jobs; ++k) {
+      const int j = two ? k : 2 * k + x;
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars[S_FULL + x], k & 1, p.wait_ns));
       if (!ok) break;
       tc_fence_after_sync();
       uint32_t sr[kBN];
-      tmem_ld_x128(tmem + lane_off + sb * kBN, sr);
-      tc_fence_before_sync();
-      mbar_arrive(&bars[S_FREE + sb]);
-
-      // keys past the end of a segment (cache or new rows) are masked out
+      tmem_ld_x128(tS, sr);
       int vcnt[4];
-      bool full = true;
-#pragma unroll
-      for (int s4 = 0; s4 < 4; ++s4) {
-        const int sub = 4 * j + s4;
-        int c;
-        if (sub < n_csub) c = min(kSub, gm.n_cache - sub * kSub);
-        else if (sub - n_csub < n_nsub) c = min(kSub, gm.n_new - (sub - n_csub) * kSub);
-        else c = 0;
-        vcnt[s4] = c;
-        full = full && (c == kSub);
-      }
-      if (!full) {
+      if (!tile_valid_counts(j, n_csub, n_nsub, gm, vcnt)) {
 #pragma unroll
         for (int c = 0; c < kBN; ++c)
           if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
@@ -410,19 +442,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       const bool need = m_new > m_run + kRescaleLog2;
       if (__any_sync(0xffffffffu, need)) {
         const float alpha = need ? ex2_approx(m_run - m_new) : 1.f;
-        if (j > 0) {
-          ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE], (j - 1) & 1, p.wait_ns));
+        if (k > 0) {
+          ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE + x], (k - 1) & 1, p.wait_ns));
           if (!ok) break;
           tc_fence_after_sync();
 #pragma unroll
           for (int ch = 0; ch < D / 32; ++ch) {
             uint32_t o[32];
-            tmem_ld_x32(tmem + lane_off + kOCol + ch * 32, o);
+            tmem_ld_x32(tO + ch * 32, o);
 #pragma unroll
             for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-            tmem_st_x32(tmem + lane_off + kOCol + ch * 32, o);
+            tmem_st_x32(tO + ch * 32, o);
           }
-          tc_fence_before_sync();
         }
         if (need) {
           l_run *= alpha;
@@ -440,49 +471,62 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         pk[c] = pack_bf16x2(a, b);
       }
       l_run += rs;
-      if (j >= 2) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars[P_FREE + sb], ((j >> 1) - 1) & 1, p.wait_ns));
-        if (!ok) break;
-      }
-      const uint32_t prow = sP + sb * 2 * kPanel + row * 128;
-#pragma unroll
-      for (int ch = 0; ch < kBN / 8; ++ch) {
-        const int pn = ch >> 3, cc = ch & 7;
-        st_shared_v4(prow + pn * kPanel + ((cc ^ (row & 7)) << 4), pk[4 * ch], pk[4 * ch + 1],
-                     pk[4 * ch + 2], pk[4 * ch + 3]);
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(&bars[P_FULL + sb]);
+      // P (bf16) overwrites the first 64 columns of this slot's S; the PV GEMM reads it from there
+      tmem_st_x64(tS, pk);
+      tc_fence_before_sync();
+      mbar_arrive(&bars[P_FULL + x]);
     }
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE], (nt - 1) & 1, p.wait_ns));
-    if (ok) {
+    if (ok && jobs > 0) ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE + x], (jobs - 1) & 1, p.wait_ns));
+    if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+    tc_fence_before_sync();
+    // split keys: slot B hands its (max, sum) to slot A, which merges both accumulators
+    float mB = -INFINITY, lB = 0.f;
+    if (!two) {
+      if (x == 1) {
+        merge_m[row] = (ok && jobs > 0) ? m_run : -INFINITY;
+        merge_l[row] = (ok && jobs > 0) ? l_run : 0.f;
+      }
+      named_barrier_sync(1, 256);
+      if (x == 0) {
+        mB = merge_m[row];
+        lB = merge_l[row];
+      }
+    }
+    if (ok && (two || x == 0)) {
       tc_fence_after_sync();
-      const int pr = mt * kBM + row;  // packed (query, head-in-group) row
+      const int pr = (qt0 + (two ? x : 0)) * kBM + row;  // packed (query, head-in-group) row
       const bool valid = pr < rows_q;
       const int qi = pr / p.grp;
       const int h = g * p.grp + (pr - qi * p.grp);
-      const float inv = 1.f / l_run;
+      const float m = fmaxf(m_run, mB);
+      const float a = (l_run > 0.f) ? ex2_approx(m_run - m) : 0.f;
+      const float b = (lB > 0.f) ? ex2_approx(mB - m) : 0.f;
+      const float lsum = a * l_run + b * lB;
+      const float inv = 1.f / lsum;
+      const float ca = a * inv, cb = b * inv;
+      const uint32_t tOB = tmem + lane_off + kOCol + D;  // slot B's accumulator (split keys)
       __nv_bfloat16* dst = p.out + ((gm.new_row + qi) * p.h_q + h) * D;
 #pragma unroll
       for (int ch = 0; ch < D / 32; ++ch) {
         uint32_t o[32];
-        tmem_ld_x32(tmem + lane_off + kOCol + ch * 32, o);
+        tmem_ld_x32(tO + ch * 32, o);
+        float f[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[c]) * ca;
+        if (!two && lB > 0.f) {
+          tmem_ld_x32(tOB + ch * 32, o);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) f[c] = fmaf(__uint_as_float(o[c]), cb, f[c]);
+        }
         if (valid) {
           uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
 #pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 w;
-            w.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv, __uint_as_float(o[8 * v + 1]) * inv);
-            w.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
-            w.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
-            w.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
-            d4[v] = w;
-          }
+          for (int v = 0; v < 4; ++v)
+            d4[v] = make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
+                               pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7]));
         }
       }
-      if (valid && p.lse) p.lse[(gm.new_row + qi) * p.h_q + h] = (m_run + log2f(l_run)) * kLn2;
-    } else {
-      record_error(p.err, SSM_ERR_TIMEOUT);
+      if (valid && p.lse) p.lse[(gm.new_row + qi) * p.h_q + h] = (m + log2f(lsum)) * kLn2;
     }
     tc_fence_before_sync();
   }
@@ -600,7 +644,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     attr_set.fetch_or(bit);
   }
   const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
-  dim3 grid(m_tiles, n_prob * h_kv);
+  dim3 grid((m_tiles + 1) / 2, n_prob * h_kv);
   attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(tq, tkc, tvc, tkn, tvn, p);
   return launch_status();
 }
