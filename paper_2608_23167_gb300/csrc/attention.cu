@@ -8,8 +8,11 @@
 //    positions and packs the queries of one GQA group into one row block,
 //    (query i, head-in-group hl) -> row i * grp + hl, so that a 128-row M tile
 //    of the tensor-core GEMM holds every query head that shares a K/V head.
-//  * attn_fwd_kernel: one CTA per (problem, kv head, pair of 128-row query
-//    tiles).  Warp 0 streams K/V tiles with TMA (128 keys = four 32-row
+//  * attn_fwd_kernel: persistent, one CTA per SM.  Work units are (problem,
+//    kv head, pair of 128-row query tiles), taken round-robin; barrier phases
+//    carry over from unit to unit, so the next unit's Q/K loads and first
+//    QK^T overlap the current unit's last softmax and epilogue.  Per unit,
+//    warp 0 streams K/V tiles with TMA (128 keys = four 32-row
 //    sub-boxes, so the cache segment and the new-row segment pack back to back
 //    with at most 31 padded keys each; 3-stage K ring, 2-stage V ring).  Warp 1
 //    issues tcgen05.mma: S = Q K^T from shared memory into tensor memory, and
@@ -23,6 +26,7 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 
@@ -49,14 +53,17 @@ constexpr uint64_t kDrainNs = 200000000ull;
 
 enum Bar {
   Q_FULL = 0,
-  K_FULL = 1,
+  Q_EMPTY = 1,
+  K_FULL = 2,
   K_EMPTY = K_FULL + kKStages,
   V_FULL = K_EMPTY + kKStages,
   V_EMPTY = V_FULL + kVStages,
   S_FULL = V_EMPTY + kVStages,  // [2]: one per slot
   P_FULL = S_FULL + 2,          // [2]
   O_DONE = P_FULL + 2,          // [2]
-  DRAIN = O_DONE + 2,
+  O_FREE = O_DONE + 2,          // [2]: the epilogue has read the slot's O
+  MERGE_FULL = O_FREE + 2,      // split keys: slot B's (max, sum) are in shared memory
+  DRAIN = MERGE_FULL + 1,
   N_BARS = DRAIN + 1
 };
 
@@ -79,6 +86,8 @@ struct AttnParams {
   int32_t n_new_u, n_cache_u;
   int32_t h_q, h_kv, grp;
   int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
+  int32_t units_per_pg;              // query-tile pairs per (problem, kv head)
+  int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)
   __nv_bfloat16* out;
   float* lse;
@@ -217,11 +226,52 @@ __device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub,
   return full;
 }
 
+// Warp-level barrier use by the softmax warps: one lane polls (so 256 threads do
+// not hammer the shared-memory pipe the MMA thread and TMA also use) and the
+// result is broadcast; arrivals are one per warp after the lanes converge.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, limit_ns);
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
+// One work unit: a pair of query tiles of one (problem, kv head).
+struct Unit {
+  Geom gm;
+  int prob, g, qt0, rows_q, n_csub, n_nsub, nt;
+  bool two, valid;
+};
+
+__device__ __forceinline__ Unit make_unit(const AttnParams& p, int u) {
+  Unit w;
+  const int pg = u / p.units_per_pg;
+  const int pair = u - pg * p.units_per_pg;
+  w.prob = pg / p.h_kv;
+  w.g = pg - w.prob * p.h_kv;
+  w.gm = problem_geom(p, w.prob);
+  w.rows_q = w.gm.n_new * p.grp;
+  const int n_qt = (w.rows_q + kBM - 1) / kBM;
+  w.qt0 = 2 * pair;
+  w.valid = w.qt0 < n_qt;
+  w.two = w.qt0 + 1 < n_qt;
+  w.n_csub = (w.gm.n_cache + kSub - 1) / kSub;
+  w.n_nsub = (w.gm.n_new + kSub - 1) / kSub;
+  w.nt = (w.n_csub + w.n_nsub + 3) / 4;
+  return w;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
     const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kn,
-    const __grid_constant__ CUtensorMap tm_vn, const AttnParams p) {
+    const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc128,
+    const __grid_constant__ CUtensorMap tm_vc128, const __grid_constant__ CUtensorMap tm_kn128,
+    const __grid_constant__ CUtensorMap tm_vn128, const AttnParams p) {
   using L = Layout<D>;
   constexpr int NP = L::NP;
   constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
@@ -231,26 +281,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + N_BARS);
-  float* merge_m = reinterpret_cast<float*>(smem + L::MERGE);
-  float* merge_l = merge_m + kBM;
+  float* merge_buf = reinterpret_cast<float*>(smem + L::MERGE);  // [m | l][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int prob = blockIdx.y / p.h_kv;
-  const int g = blockIdx.y - prob * p.h_kv;
-  const Geom gm = problem_geom(p, prob);
-  const int rows_q = gm.n_new * p.grp;
-  const int n_qt = (rows_q + kBM - 1) / kBM;
-  const int qt0 = 2 * blockIdx.x;            // first query tile of this CTA
-  if (qt0 >= n_qt) return;                   // whole CTA, before any shared state exists
-  const bool two = qt0 + 1 < n_qt;           // two query tiles, else the slots split the keys
   const bool uniform = p.problems == nullptr;
-  const int n_csub = (gm.n_cache + kSub - 1) / kSub;
-  const int n_nsub = (gm.n_new + kSub - 1) / kSub;
-  const int nt = (n_csub + n_nsub + 3) / 4;  // key tiles
-  const int n_jobs = two ? 2 * nt : nt;      // job t: slot t & 1, key tile two ? t >> 1 : t
 
   if (threadIdx.x == 0) {
     mbar_init(&bars[Q_FULL], 1);
+    mbar_init(&bars[Q_EMPTY], 1);
     for (int s = 0; s < kKStages; ++s) {
       mbar_init(&bars[K_FULL + s], 1);
       mbar_init(&bars[K_EMPTY + s], 1);
@@ -261,9 +299,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&bars[S_FULL + x], 1);
-      mbar_init(&bars[P_FULL + x], 128);
+      mbar_init(&bars[P_FULL + x], 4);   // one arrival per softmax warp
       mbar_init(&bars[O_DONE + x], 1);
+      mbar_init(&bars[O_FREE + x], 4);
     }
+    mbar_init(&bars[MERGE_FULL], 4);
     mbar_init(&bars[DRAIN], 1);
     fence_mbar_init();
   }
@@ -287,124 +327,167 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
-      int last_k = -1, last_v = -1;  // latest K / V tile whose load was issued
-      const int nq = two ? 2 : 1;
-      mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
-      for (int x = 0; x < nq; ++x) {
-        int qy, qz;
-        if (uniform) {
-          qy = (qt0 + x) * kBM;
-          qz = prob * p.h_kv + g;
-        } else {
-          qy = static_cast<int>((gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp) + (qt0 + x) * kBM;
-          qz = 0;
-        }
-#pragma unroll
-        for (int pn = 0; pn < NP; ++pn)
-          tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
-      }
-      const int c3 = uniform ? prob : 0;
-      // K runs one tile ahead of V: K(j) then V(j - 1)
-      for (int j = 0; j <= nt && ok; ++j) {
-        for (int half = 0; half < 2 && ok; ++half) {
-          const int jt = half ? j - 1 : j;
-          if (jt < 0 || jt >= nt) continue;
-          const int nst = half ? kVStages : kKStages;
-          const int st = jt % nst;
-          const int fill = jt / nst;
-          if (fill > 0) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
-          if (!ok) break;
-          uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
-          mbar_arrive_expect_tx(full, L::TILE);
-          uint8_t* dst = smem + (half ? L::V : L::K) + st * L::TILE;
-#pragma unroll
-          for (int sb = 0; sb < 4; ++sb) {
-            const int sub = 4 * jt + sb;
-            const CUtensorMap* map;
-            int c2;
-            if (sub < n_csub) {
-              map = half ? &tm_vc : &tm_kc;
-              c2 = uniform ? sub * kSub : static_cast<int>(gm.cache_row + sub * kSub);
-            } else if (sub - n_csub < n_nsub) {
-              map = half ? &tm_vn : &tm_kn;
-              c2 = uniform ? (sub - n_csub) * kSub : static_cast<int>(gm.new_row + (sub - n_csub) * kSub);
-            } else {
-              map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
-              c2 = p.new_rows_extent;
-            }
-#pragma unroll
-            for (int pn = 0; pn < NP; ++pn)
-              tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, g, c2, c3);
+      int qcount = 0;            // units whose Q was loaded
+      int kfill = 0, vfill = 0;  // K / V tiles loaded so far (all units)
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, u);
+        if (!w.valid) continue;
+        if (qcount > 0) ok = mbar_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
+        if (!ok) break;
+        const int nq = w.two ? 2 : 1;
+        mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
+        for (int x = 0; x < nq; ++x) {
+          int qy, qz;
+          if (uniform) {
+            qy = (w.qt0 + x) * kBM;
+            qz = w.prob * p.h_kv + w.g;
+          } else {
+            qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
+                 (w.qt0 + x) * kBM;
+            qz = 0;
           }
-          if (half) last_v = jt;
-          else last_k = jt;
+#pragma unroll
+          for (int pn = 0; pn < NP; ++pn)
+            tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+        }
+        ++qcount;
+        const int c3 = uniform ? w.prob : 0;
+        // K runs one tile ahead of V: K(j) then V(j - 1)
+        for (int j = 0; j <= w.nt && ok; ++j) {
+          for (int half = 0; half < 2 && ok; ++half) {
+            const int jt = half ? j - 1 : j;
+            if (jt < 0 || jt >= w.nt) continue;
+            const int nst = half ? kVStages : kKStages;
+            const int idx = half ? vfill : kfill;
+            const int st = idx % nst, fill = idx / nst;
+            if (fill > 0) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
+            if (!ok) break;
+            uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
+            mbar_arrive_expect_tx(full, L::TILE);
+            uint8_t* dst = smem + (half ? L::V : L::K) + st * L::TILE;
+            const int sub0 = 4 * jt;
+            const bool whole_cache = sub0 + 3 < w.n_csub && (sub0 + 4) * kSub <= w.gm.n_cache;
+            const bool whole_new = sub0 >= w.n_csub && (sub0 - w.n_csub + 4) * kSub <= w.gm.n_new;
+            if (whole_cache || whole_new) {
+              const CUtensorMap* map = whole_cache ? (half ? &tm_vc128 : &tm_kc128) : (half ? &tm_vn128 : &tm_kn128);
+              const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
+                                         : (uniform ? (sub0 - w.n_csub) * kSub
+                                                    : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
+#pragma unroll
+              for (int pn = 0; pn < NP; ++pn) tma_load_4d(dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
+            } else
+#pragma unroll
+            for (int sb = 0; sb < 4; ++sb) {
+              const int sub = 4 * jt + sb;
+              const CUtensorMap* map;
+              int c2;
+              if (sub < w.n_csub) {
+                map = half ? &tm_vc : &tm_kc;
+                c2 = uniform ? sub * kSub : static_cast<int>(w.gm.cache_row + sub * kSub);
+              } else if (sub - w.n_csub < w.n_nsub) {
+                map = half ? &tm_vn : &tm_kn;
+                c2 = uniform ? (sub - w.n_csub) * kSub : static_cast<int>(w.gm.new_row + (sub - w.n_csub) * kSub);
+              } else {
+                map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
+                c2 = p.new_rows_extent;
+              }
+#pragma unroll
+              for (int pn = 0; pn < NP; ++pn)
+                tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
+            }
+            if (half) ++vfill;
+            else ++kfill;
+          }
         }
       }
       if (!ok) {
         record_error(p.err, SSM_ERR_TIMEOUT);
         // let every copy in flight land before the CTA's shared memory is released:
         // the newest fill of each stage is the only one that can still be in flight
-        mbar_wait(&bars[Q_FULL], 0, kDrainNs);
-        for (int jt = max(0, last_k - kKStages + 1); jt <= last_k; ++jt)
-          mbar_wait(&bars[K_FULL + jt % kKStages], (jt / kKStages) & 1, kDrainNs);
-        for (int jt = max(0, last_v - kVStages + 1); jt <= last_v; ++jt)
-          mbar_wait(&bars[V_FULL + jt % kVStages], (jt / kVStages) & 1, kDrainNs);
+        if (qcount > 0) mbar_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
+        for (int i = max(0, kfill - kKStages); i < kfill; ++i)
+          mbar_wait(&bars[K_FULL + i % kKStages], (i / kKStages) & 1, kDrainNs);
+        for (int i = max(0, vfill - kVStages); i < vfill; ++i)
+          mbar_wait(&bars[V_FULL + i % kVStages], (i / kVStages) & 1, kDrainNs);
       }
     }
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      bool ok = mbar_wait(&bars[Q_FULL], 0, p.wait_ns);
-      tc_fence_after_sync();
-      const uint32_t sQ = smem_u32(smem + L::Q);
-      const uint32_t sK = smem_u32(smem + L::K);
-      const uint32_t sV = smem_u32(smem + L::V);
-      int kx0 = 0, kx1 = 0;        // jobs issued per slot
-      int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
-      // O_X += P_X V(j) for slot X's latest job
-      auto issue_pv = [&](int x) -> bool {
-        const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
-        if (!mbar_wait(&bars[P_FULL + x], k & 1, p.wait_ns)) return false;
-        if (!mbar_wait(&bars[V_FULL + jp % kVStages], (jp / kVStages) & 1, p.wait_ns)) return false;
-        tc_fence_after_sync();
-        const uint32_t vb = sV + (jp % kVStages) * L::TILE;
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk)
-          umma_bf16_ts(tmem + kOCol + x * D, tmem + x * kBN + kk * 8, sdesc_sw128(vb + kk * 16 * 128, kPanel, 1024),
-                       kIdescPV, (k > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&bars[O_DONE + x]);
-        if (!two || x == 1) umma_commit(&bars[V_EMPTY + jp % kVStages]);
-        return true;
-      };
-      for (int t = 0; t < n_jobs && ok; ++t) {
-        const int x = t & 1;
-        const int j = two ? (t >> 1) : t;
-        if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
+      bool ok = true;
+      // operand descriptors: the per-instruction ones differ only in the start address field
+      const uint64_t dQ = sdesc_sw128(smem_u32(smem + L::Q), 16, 1024);
+      const uint64_t dK = sdesc_sw128(smem_u32(smem + L::K), 16, 1024);
+      const uint64_t dV = sdesc_sw128(smem_u32(smem + L::V), kPanel, 1024);
+      int ucount = 0;            // units processed
+      int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
+      int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, u);
+        if (!w.valid) continue;
+        ok = mbar_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
         if (!ok) break;
-        ok = mbar_wait(&bars[K_FULL + j % kKStages], (j / kKStages) & 1, p.wait_ns);
-        if (!ok) break;
-        tc_fence_after_sync();
-        const uint32_t qb = sQ + (two ? x : 0) * L::TILE;
-        const uint32_t kb = sK + (j % kKStages) * L::TILE;
+        int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
+        int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
+        bool freed0 = false, freed1 = false;
+        // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O
+        auto wait_o_free = [&](int x) -> bool {
+          bool& f = x ? freed1 : freed0;
+          if (f) return true;
+          f = true;
+          return ucount == 0 || mbar_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
+        };
+        // O_X += P_X V(j) for slot X's latest job
+        auto issue_pv = [&](int x) -> bool {
+          const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
+          int& pv = x ? pv1 : pv0;
+          if (!wait_o_free(x)) return false;
+          if (!mbar_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
+          const int vi = vbase + jp;
+          if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
+          tc_fence_after_sync();
+          const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
+          const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
+          const uint32_t acc0 = k > 0 ? 1u : 0u;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
-          umma_bf16_ss(tmem + x * kBN, sdesc_sw128(qb + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024), kIdescQK,
-                       kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            umma_bf16_ts(d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4), kIdescPV,
+                         kk > 0 ? 1u : acc0);
+          umma_commit(&bars[O_DONE + x]);
+          if (!w.two || x == 1) umma_commit(&bars[V_EMPTY + vi % kVStages]);
+          ++pv;
+          return true;
+        };
+        const int n_jobs = w.two ? 2 * w.nt : w.nt;
+        for (int t = 0; t < n_jobs && ok; ++t) {
+          const int x = t & 1;
+          const int j = w.two ? (t >> 1) : t;
+          if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
+          if (!ok) break;
+          const int ki = kbase + j;
+          ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
+          if (!ok) break;
+          const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
+          const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
+          const uint32_t s_tmem = tmem + x * kBN;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
+            umma_bf16_ss(s_tmem, qb + off, kb + off, kIdescQK, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(&bars[S_FULL + x]);
+          if (!w.two || x == 1) umma_commit(&bars[K_EMPTY + ki % kKStages]);
+          if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
         }
-        umma_commit(&bars[S_FULL + x]);
-        if (!two || x == 1) umma_commit(&bars[K_EMPTY + j % kKStages]);
-        if (x) {
-          jlast1 = j;
-          ++kx1;
-        } else {
-          jlast0 = j;
-          ++kx0;
-        }
+        if (ok) umma_commit(&bars[Q_EMPTY]);
+        if (ok && kx0 > 0) ok = issue_pv(0);
+        if (ok && kx1 > 0) ok = issue_pv(1);
+        if (ok) ok = wait_o_free(0) && wait_o_free(1);
+        kbase += w.nt;
+        vbase += w.nt;
+        ++ucount;
       }
-      if (ok && kx0 > 0) ok = issue_pv(0);
-      if (ok && kx1 > 0) ok = issue_pv(1);
       if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
       // every issued MMA completes before tensor memory is released
       umma_commit(&bars[DRAIN]);
@@ -419,115 +502,140 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const uint32_t tS = tmem + lane_off + x * kBN;
     const uint32_t tO = tmem + lane_off + kOCol + x * D;
-    const int jobs = two ? nt : (x == 0 ? (nt + 1) / 2 : nt / 2);
-    float m_run = -INFINITY, l_run = 0.f;
+    const uint32_t tOB = tmem + lane_off + kOCol + D;  // slot B's accumulator (split keys)
     bool ok = true;
-    for (int k = 0; k < jobs; ++k) {
-      const int j = two ? k : 2 * k + x;
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars[S_FULL + x], k & 1, p.wait_ns));
-      if (!ok) break;
-      tc_fence_after_sync();
-      uint32_t sr[kBN];
-      tmem_ld_x128(tS, sr);
-      int vcnt[4];
-      if (!tile_valid_counts(j, n_csub, n_nsub, gm, vcnt)) {
+    int sj = 0;       // S tiles consumed by this slot (all units)
+    int merges = 0;   // split-key merges done
+    for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+      const Unit w = make_unit(p, u);
+      if (!w.valid) continue;
+      const int jobs = w.two ? w.nt : (x == 0 ? (w.nt + 1) / 2 : w.nt / 2);
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int k = 0; k < jobs; ++k) {
+        const int j = w.two ? k : 2 * k + x;
+        ok = warp_wait(&bars[S_FULL + x], sj & 1, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after_sync();
+        uint32_t sr[kBN];
+        tmem_ld_x128(tS, sr);
+        int vcnt[4];
+        if (!tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, vcnt)) {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c)
-          if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
-      }
-      float mx = -INFINITY;
+          for (int c = 0; c < kBN; ++c)
+            if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
+        }
+        // row maximum: eight independent chains of 3-input max, then a short tree
+        float mx8[8];
 #pragma unroll
-      for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, __uint_as_float(sr[c]));
-      const float m_new = fmaxf(m_run, mx * p.scale_log2);
-      const bool need = m_new > m_run + kRescaleLog2;
-      if (__any_sync(0xffffffffu, need)) {
-        const float alpha = need ? ex2_approx(m_run - m_new) : 1.f;
-        if (k > 0) {
-          ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE + x], (k - 1) & 1, p.wait_ns));
-          if (!ok) break;
-          tc_fence_after_sync();
+        for (int c = 0; c < 8; ++c) mx8[c] = __uint_as_float(sr[c]);
 #pragma unroll
-          for (int ch = 0; ch < D / 32; ++ch) {
-            uint32_t o[32];
-            tmem_ld_x32(tO + ch * 32, o);
+        for (int c = 8; c < kBN; c += 2)
+          mx8[(c >> 1) & 7] = fmax3(mx8[(c >> 1) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
+        const float mx = fmaxf(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7]));
+        const float m_new = fmaxf(m_run, mx * p.scale_log2);
+        const bool need = m_new > m_run + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = need ? ex2_approx(m_run - m_new) : 1.f;
+          if (k > 0) {
+            // the previous PV of this slot completed before this S tile was committed
+            ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
+            if (!ok) break;
+            tc_fence_after_sync();
 #pragma unroll
-            for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-            tmem_st_x32(tO + ch * 32, o);
+            for (int ch = 0; ch < D / 32; ++ch) {
+              uint32_t o[32];
+              tmem_ld_x32(tO + ch * 32, o);
+#pragma unroll
+              for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+              tmem_st_x32(tO + ch * 32, o);
+            }
+          }
+          if (need) {
+            l_run *= alpha;
+            m_run = m_new;
           }
         }
-        if (need) {
-          l_run *= alpha;
-          m_run = m_new;
-        }
-      }
-      const float neg = -m_run;
-      float rs = 0.f;
-      uint32_t pk[kBN / 2];
+        // p = 2^(s * scale * log2 e - m): packed pair FMA, two MUFU ex2, packed pair sums
+        const float neg = -m_run, sc = p.scale_log2;
+        float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
+        uint32_t pk[kBN / 2];
 #pragma unroll
-      for (int c = 0; c < kBN / 2; ++c) {
-        const float a = ex2_approx(fmaf(__uint_as_float(sr[2 * c]), p.scale_log2, neg));
-        const float b = ex2_approx(fmaf(__uint_as_float(sr[2 * c + 1]), p.scale_log2, neg));
-        rs += a + b;
-        pk[c] = pack_bf16x2(a, b);
+        for (int c = 0; c < kBN / 2; ++c) {
+          float t0, t1;
+          ffma2(t0, t1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), sc, sc, neg, neg);
+          const float a = ex2_approx(t0), b = ex2_approx(t1);
+          fadd2_acc(ra[c & 3], rb[c & 3], a, b);
+          pk[c] = pack_bf16x2(a, b);
+        }
+        l_run += ((ra[0] + rb[0]) + (ra[1] + rb[1])) + ((ra[2] + rb[2]) + (ra[3] + rb[3]));
+        // P (bf16) overwrites the first 64 columns of this slot's S; the PV GEMM reads it from there
+        tmem_st_x64(tS, pk);
+        tc_fence_before_sync();
+        warp_arrive(&bars[P_FULL + x]);
+        ++sj;
       }
-      l_run += rs;
-      // P (bf16) overwrites the first 64 columns of this slot's S; the PV GEMM reads it from there
-      tmem_st_x64(tS, pk);
-      tc_fence_before_sync();
-      mbar_arrive(&bars[P_FULL + x]);
-    }
-    if (ok && jobs > 0) ok = __all_sync(0xffffffffu, mbar_wait(&bars[O_DONE + x], (jobs - 1) & 1, p.wait_ns));
-    if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
-    tc_fence_before_sync();
-    // split keys: slot B hands its (max, sum) to slot A, which merges both accumulators
-    float mB = -INFINITY, lB = 0.f;
-    if (!two) {
-      if (x == 1) {
-        merge_m[row] = (ok && jobs > 0) ? m_run : -INFINITY;
-        merge_l[row] = (ok && jobs > 0) ? l_run : 0.f;
-      }
-      named_barrier_sync(1, 256);
-      if (x == 0) {
-        mB = merge_m[row];
-        lB = merge_l[row];
-      }
-    }
-    if (ok && (two || x == 0)) {
+      // the slot's last PV of this unit (it completes before any later S of this slot)
+      if (ok && jobs > 0) ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
+      if (!ok) break;
       tc_fence_after_sync();
-      const int pr = (qt0 + (two ? x : 0)) * kBM + row;  // packed (query, head-in-group) row
-      const bool valid = pr < rows_q;
-      const int qi = pr / p.grp;
-      const int h = g * p.grp + (pr - qi * p.grp);
-      const float m = fmaxf(m_run, mB);
-      const float a = (l_run > 0.f) ? ex2_approx(m_run - m) : 0.f;
-      const float b = (lB > 0.f) ? ex2_approx(mB - m) : 0.f;
-      const float lsum = a * l_run + b * lB;
-      const float inv = 1.f / lsum;
-      const float ca = a * inv, cb = b * inv;
-      const uint32_t tOB = tmem + lane_off + kOCol + D;  // slot B's accumulator (split keys)
-      __nv_bfloat16* dst = p.out + ((gm.new_row + qi) * p.h_q + h) * D;
-#pragma unroll
-      for (int ch = 0; ch < D / 32; ++ch) {
-        uint32_t o[32];
-        tmem_ld_x32(tO + ch * 32, o);
-        float f[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[c]) * ca;
-        if (!two && lB > 0.f) {
-          tmem_ld_x32(tOB + ch * 32, o);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) f[c] = fmaf(__uint_as_float(o[c]), cb, f[c]);
+      // split keys: slot B hands its (max, sum) to slot A, which merges both accumulators
+      // Split keys: slot B hands its (max, sum) to slot A, which merges both accumulators.
+      // The buffer is rewritten only after slot B's last PV of a later unit, which the MMA
+      // issues after slot A freed this unit's accumulators, i.e. after slot A's reads.
+      float mB = -INFINITY, lB = 0.f;
+      if (!w.two && w.nt >= 2) {
+        if (x == 1) {
+          merge_buf[row] = m_run;
+          merge_buf[kBM + row] = l_run;
+          warp_arrive(&bars[MERGE_FULL]);
+        } else {
+          ok = warp_wait(&bars[MERGE_FULL], merges & 1, p.wait_ns);
+          if (!ok) break;
+          mB = merge_buf[row];
+          lB = merge_buf[kBM + row];
         }
-        if (valid) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
-#pragma unroll
-          for (int v = 0; v < 4; ++v)
-            d4[v] = make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
-                               pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7]));
-        }
+        ++merges;
       }
-      if (valid && p.lse) p.lse[(gm.new_row + qi) * p.h_q + h] = (m + log2f(lsum)) * kLn2;
+      if (w.two || x == 0) {
+        const int pr = (w.qt0 + (w.two ? x : 0)) * kBM + row;  // packed (query, head-in-group) row
+        const bool valid = pr < w.rows_q;
+        const int qi = pr / p.grp;
+        const int h = w.g * p.grp + (pr - qi * p.grp);
+        const float m = fmaxf(m_run, mB);
+        const float a = (l_run > 0.f) ? ex2_approx(m_run - m) : 0.f;
+        const float b = (lB > 0.f) ? ex2_approx(mB - m) : 0.f;
+        const float lsum = a * l_run + b * lB;
+        const float inv = 1.f / lsum;
+        const float ca = a * inv, cb = b * inv;
+        __nv_bfloat16* dst = p.out + ((w.gm.new_row + qi) * p.h_q + h) * D;
+#pragma unroll
+        for (int ch = 0; ch < D / 32; ++ch) {
+          uint32_t o[32];
+          tmem_ld_x32(tO + ch * 32, o);
+          float f[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[c]) * ca;
+          if (!w.two && lB > 0.f) {
+            tmem_ld_x32(tOB + ch * 32, o);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) f[c] = fmaf(__uint_as_float(o[c]), cb, f[c]);
+          }
+          if (valid) {
+            uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              d4[v] = make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
+                                 pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7]));
+          }
+        }
+        if (valid && p.lse) p.lse[(w.gm.new_row + qi) * p.h_q + h] = (m + log2f(lsum)) * kLn2;
+        // this slot's O (and, with split keys, slot B's O too) may now be overwritten
+        tc_fence_before_sync();
+        warp_arrive(&bars[O_FREE + x]);
+        if (!w.two) warp_arrive(&bars[O_FREE + 1]);
+      }
     }
+    if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
     tc_fence_before_sync();
   }
   __syncthreads();
@@ -588,7 +696,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   auto* qhat = static_cast<__nv_bfloat16*>(workspace);
   auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) +
                                                 align_up(static_cast<size_t>(total_new) * h_q * D * 2, 256));
-  CUtensorMap tq, tkc, tvc, tkn, tvn;
+  CUtensorMap tq, tkc, tvc, tkn, tvn, tkc128, tvc128, tkn128, tvn128;
   {
     const uint64_t dq[3] = {static_cast<uint64_t>(D),
                             static_cast<uint64_t>(uniform ? new_rows_per_b * grp : total_new * h_q),
@@ -600,14 +708,21 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                             static_cast<uint64_t>(new_rows_per_b), static_cast<uint64_t>(nb)};
     if (!make_map(&tkn, khat, 4, dn, bkv)) return SSM_ERR_CUDA;
     if (!make_map(&tvn, v_new, 4, dn, bkv)) return SSM_ERR_CUDA;
+    const uint32_t bkv128[4] = {64, 1, kBN, 1};
+    if (!make_map(&tkn128, khat, 4, dn, bkv128)) return SSM_ERR_CUDA;
+    if (!make_map(&tvn128, v_new, 4, dn, bkv128)) return SSM_ERR_CUDA;
     if (cache_rows_per_b > 0) {
       const uint64_t dc[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
                               static_cast<uint64_t>(cache_rows_per_b), static_cast<uint64_t>(nb)};
       if (!make_map(&tkc, k_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
       if (!make_map(&tvc, v_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
+      if (!make_map(&tkc128, k_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
+      if (!make_map(&tvc128, v_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
     } else {
       tkc = tkn;  // never read: no problem has cache rows
       tvc = tvn;
+      tkc128 = tkn128;
+      tvc128 = tvn128;
     }
   }
   AttnParams p{};
@@ -644,8 +759,12 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     attr_set.fetch_or(bit);
   }
   const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
-  dim3 grid((m_tiles + 1) / 2, n_prob * h_kv);
-  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(tq, tkc, tvc, tkn, tvn, p);
+  p.units_per_pg = (m_tiles + 1) / 2;
+  const int64_t total_units = static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
+  if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
+  p.total_units = static_cast<int32_t>(total_units);
+  const int grid = static_cast<int>(std::min<int64_t>(total_units, num_sms()));
+  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(tq, tkc, tvc, tkn, tvn, tkc128, tvc128, tkn128, tvn128, p);
   return launch_status();
 }
 
