@@ -173,7 +173,8 @@ class StepInputs:
                                  workspace=self.attn_ws)
         if ev is not None:
             ev[3].record()
-        ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=self.p2,
+        # the threshold rule needs no second-largest probability, so p2 is not requested
+        ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=None,
                        threshold=w.threshold, min_commit=1, workspace=self.unmask_ws)
         if ev is not None:
             ev[4].record()

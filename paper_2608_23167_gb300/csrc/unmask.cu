@@ -1,25 +1,34 @@
 // unmask.cu -- confidence-based unmasking (Sec. 4.1 "Baselines": Vanilla top-1
 // and parallel threshold decoding; Sec. 4.5: margin decoding).
 //
-// Pass 1 (unmask_partial_kernel): every masked row of logits is cut into
-// chunks; one CTA reads one chunk once with 16-byte loads and reduces it to
-// (max, sum of exp(x - max), first argmax, second-largest logit).  The grid is
-// chunks x rows, so a 126464-entry bf16 row spreads over 16 CTAs and the whole
-// read is spread evenly over the SMs.  Pass 2 (unmask_commit_kernel): one CTA
-// per batch row merges the chunk partials of its positions, writes conf /
+// Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
+// segments of 32768 entries (the work items, dealt round-robin to persistent
+// CTAs, six per SM).  Each thread streams its own 64-byte slices of successive
+// 16 KB chunks from HBM into a private two-stage shared-memory ring with
+// 16-byte cp.async copies, so the read runs ahead of the arithmetic without any
+// barrier (a thread only reads back what it copied itself), and folds every
+// chunk into a running (max, first argmax, sum of exp(x - max)) plus, when p2
+// is wanted, the second-largest value.  The 256 running states of a segment are
+// merged into one partial.  Rows whose length or alignment rules out 16-byte
+// copies take unmask_partial_scalar_kernel on the same segment grid.
+// Pass 2 (unmask_commit_kernel): one CTA
+// per batch row merges the segment partials of its positions, writes conf /
 // argmax / p2 and applies the commit rule.  Logits of unmasked rows are never
 // read.
 #include <cuda_bf16.h>
 
+#include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
+#include "sm100_ptx.cuh"
 
 namespace ssm {
 namespace {
 
 constexpr int kUnmaskThreads = 256;
-constexpr int kUnroll = 16;                        // 16-byte vectors per thread per chunk
+constexpr int kUnroll = 16;                        // a segment is 256 x 16 vectors of 16 bytes
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Partial {
@@ -102,104 +111,204 @@ struct Vec<float> {
   __device__ static float scalar(const float* p, int64_t i) { return p[i]; }
 };
 
-// Block-wide reductions over the 256 threads of a CTA (result in every thread).
-__device__ __forceinline__ float block_max(float v, float* red) {
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, d));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  v = red[lane & (kUnmaskThreads / 32 - 1)];
-#pragma unroll
-  for (int d = kUnmaskThreads / 64; d >= 1; d >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, d));
-  return v;
+// ---------------------------------------------------------------------------
+// Streaming pass: bulk copies into a shared-memory ring, 8 consumer warps
+// ---------------------------------------------------------------------------
+
+constexpr int kStreamThreads = 256;
+constexpr int kStageBytes = 16384;                     // one stage: 64 bytes per thread
+constexpr int kStreamStages = 2;                       // chunks in flight per thread
+constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
+
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("min.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ float lo_bf16(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float hi_bf16(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// 16-byte asynchronous global -> shared copy (L2 only, bypassing L1).
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// Chunk of one row: thread t holds vectors t, t + 256, ..., t + 256 (U - 1) of
-// the chunk (16 bytes each, so a warp reads 512 contiguous bytes per vector).
-// Pass 1 keeps the two largest values per thread; after the block maximum M is
-// known, pass 2 sums exp(x - M) and the holder(s) of M report its first index.
-template <typename T, int U>
-__global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_vec_kernel(
-    const T* __restrict__ logits, int64_t vocab, int64_t chunk, int n_chunks,
-    const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
-  constexpr int N = Vec<T>::N;
-  __shared__ float red_f[kUnmaskThreads / 32];
-  __shared__ Partial red_p[kUnmaskThreads / 32];
-  const int64_t row = blockIdx.y;
-  if (!masked[row]) return;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * chunk;
-  const int64_t c1 = min(vocab, c0 + chunk);
-  const uint4* xv = reinterpret_cast<const uint4*>(logits + row * vocab);
-  uint4 v[U];
-#pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
-    v[u] = (e < c1) ? __ldcs(xv + e / N) : make_uint4(0, 0, 0, 0);
-  }
-  float m1 = -INFINITY, m2 = -INFINITY;
-#pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
-    if (e < c1) {
-      float f[N];
-      Vec<T>::unpack(v[u], f);
-#pragma unroll
-      for (int c = 0; c < N; ++c) {
-        m2 = fmaxf(m2, fminf(m1, f[c]));
-        m1 = fmaxf(m1, f[c]);
-      }
+// Walks the chunks of this CTA's work items (masked rows only) in order.
+struct ChunkIter {
+  int64_t item, off, bytes, e0, row;
+  bool valid;
+};
+
+// Running per-thread state over one segment: max m1 (first index idx), second
+// largest m2 (a repeated maximum counts twice) and s = sum exp(x - m1).
+struct RunState {
+  float m1, m2, s;
+  int idx;
+};
+
+template <typename T>
+__device__ __forceinline__ void chunk_seek(ChunkIter& it, int64_t vocab, int64_t seg_elems, int n_seg,
+                                           int64_t n_items, const uint8_t* __restrict__ masked) {
+  // advance to the next item that has a masked row, if the current one is exhausted
+  while (it.item < n_items && (it.off >= it.bytes)) {
+    it.item += gridDim.x;
+    it.off = 0;
+    if (it.item >= n_items) break;
+    it.row = it.item / n_seg;
+    if (!masked[it.row]) {
+      it.bytes = 0;
+      continue;
     }
+    it.e0 = (it.item - it.row * n_seg) * seg_elems;
+    it.bytes = (min(vocab, it.e0 + seg_elems) - it.e0) * static_cast<int64_t>(sizeof(T));
   }
-  const float M = block_max(m1, red_f);
-  const float mb = (M == -INFINITY) ? 0.f : M * kLog2e;  // a chunk of -inf logits sums to 0
-  float s = 0.f;
-  int idx = INT_MAX;
-#pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int64_t e = c0 + (static_cast<int64_t>(u) * kUnmaskThreads + threadIdx.x) * N;
-    if (e < c1) {
-      float f[N];
-      Vec<T>::unpack(v[u], f);
-#pragma unroll
-      for (int c = 0; c < N; ++c) s += ex2(fmaf(f[c], kLog2e, -mb));
-      if (m1 == M && idx == INT_MAX) {
-#pragma unroll
-        for (int c = 0; c < N; ++c)
-          if (f[c] == M && idx == INT_MAX) idx = static_cast<int>(e + c);
-      }
-    }
-  }
-  // (m, s, idx, second): a thread whose maximum is below M offers it as a second
-  // candidate; two threads holding M make M itself the second-largest value.
-  Partial p{M, s, idx, (m1 == M) ? m2 : m1};
-  int holders = (m1 == M) ? 1 : 0;
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) {
-    p.s += __shfl_xor_sync(0xffffffffu, p.s, d);
-    p.idx = min(p.idx, __shfl_xor_sync(0xffffffffu, p.idx, d));
-    p.m2 = fmaxf(p.m2, __shfl_xor_sync(0xffffffffu, p.m2, d));
-    holders += __shfl_xor_sync(0xffffffffu, holders, d);
-  }
+  it.valid = it.item < n_items;
+}
+
+template <typename T, bool NEED_SECOND>
+__global__ void __launch_bounds__(kStreamThreads) unmask_stream_kernel(
+    const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
+    const uint8_t* __restrict__ masked, Partial* __restrict__ part, unsigned* err, uint64_t wait_ns) {
+  constexpr int ESZ = sizeof(T);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+  __shared__ Partial wpart[kStreamThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) {
-    p.m = __int_as_float(holders);  // the warp's holder count rides in the unused m field
-    red_p[warp] = p;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    Partial q = red_p[lane & (kUnmaskThreads / 32 - 1)];
-    int h = (lane < kUnmaskThreads / 32) ? __float_as_int(q.m) : 0;
-    if (lane >= kUnmaskThreads / 32) q = Partial{0.f, 0.f, INT_MAX, -INFINITY};
+  const int64_t n_items = n_rows * n_seg;
+  // issue side runs kStreamStages chunks ahead of the compute side; a thread only ever
+  // reads the shared-memory bytes it copied itself, so no barrier is needed between them
+  ChunkIter is{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
+  chunk_seek<T>(is, vocab, seg_elems, n_seg, n_items, masked);
+  auto issue = [&](int slot) {
+    if (is.valid) {
+      const uint8_t* src = reinterpret_cast<const uint8_t*>(logits + is.row * vocab + is.e0) + is.off;
+      uint8_t* dst = ring + slot * kStageBytes;
 #pragma unroll
-    for (int d = kUnmaskThreads / 64; d >= 1; d >>= 1) {
-      q.s += __shfl_xor_sync(0xffffffffu, q.s, d);
-      q.idx = min(q.idx, __shfl_xor_sync(0xffffffffu, q.idx, d));
-      q.m2 = fmaxf(q.m2, __shfl_xor_sync(0xffffffffu, q.m2, d));
-      h += __shfl_xor_sync(0xffffffffu, h, d);
+      for (int u = 0; u < kVecPerThread; ++u) {
+        const int vi = u * kStreamThreads + threadIdx.x;
+        if (vi * 16 < is.bytes - is.off) cp_async16(dst + vi * 16, src + vi * 16);
+      }
+      is.off += kStageBytes;
+      chunk_seek<T>(is, vocab, seg_elems, n_seg, n_items, masked);
     }
-    if (lane == 0) part[row * n_chunks + blockIdx.x] = Partial{M, q.s, q.idx, (h >= 2) ? M : q.m2};
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int k = 0; k < kStreamStages; ++k) issue(k);
+
+  ChunkIter cs{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
+  chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
+  int slot = 0;
+  while (cs.valid) {
+    const int64_t item = cs.item;
+    const int64_t e0 = cs.e0;
+    RunState r{-INFINITY, -INFINITY, 0.f, INT_MAX};
+    while (cs.valid && cs.item == item) {
+      cp_async_wait<kStreamStages - 1>();
+      const int chunk_bytes = static_cast<int>(min(static_cast<int64_t>(kStageBytes), cs.bytes - cs.off));
+      const uint4* sv = reinterpret_cast<const uint4*>(ring + slot * kStageBytes);
+      uint4 v[kVecPerThread];
+      bool in[kVecPerThread];
+      const uint32_t ninf = (ESZ == 2) ? 0xFF80FF80u : 0xFF800000u;
+#pragma unroll
+      for (int u = 0; u < kVecPerThread; ++u) {
+        const int vi = u * kStreamThreads + threadIdx.x;
+        in[u] = vi * 16 < chunk_bytes;
+        v[u] = in[u] ? sv[vi] : make_uint4(ninf, ninf, ninf, ninf);
+      }
+      const int64_t base = e0 + cs.off / ESZ;
+      // this thread's values of the chunk as fp32 (entries past a short last chunk are -inf)
+      constexpr int PER = kVecPerThread * 16 / ESZ;  // 32 bf16 or 16 fp32 values
+      float f[PER];
+#pragma unroll
+      for (int u = 0; u < kVecPerThread; ++u) {
+        const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if constexpr (ESZ == 2) {
+            f[u * 8 + 2 * q] = lo_bf16(w4[q]);
+            f[u * 8 + 2 * q + 1] = hi_bf16(w4[q]);
+          } else {
+            f[u * 4 + q] = __uint_as_float(w4[q]);
+          }
+        }
+      }
+      // chunk maximum (four chains of 3-input max) and, when asked for, the second largest
+      float c4[4] = {f[0], f[1], f[2], f[3]};
+#pragma unroll
+      for (int e = 4; e < PER; e += 8) {
+        c4[0] = fmax3(c4[0], f[e], f[e + 1]);
+        c4[1] = fmax3(c4[1], f[e + 2], f[e + 3]);
+        if (e + 4 < PER) {
+          c4[2] = fmax3(c4[2], f[e + 4], f[e + 5]);
+          c4[3] = fmax3(c4[3], f[e + 6], f[e + 7]);
+        }
+      }
+      const float cm1 = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
+      if constexpr (NEED_SECOND) {
+        float s2 = -INFINITY, m1l = -INFINITY;
+#pragma unroll
+        for (int e = 0; e < PER; ++e) {
+          s2 = fmaxf(s2, fminf(m1l, f[e]));
+          m1l = fmaxf(m1l, f[e]);
+        }
+        // second largest of the running values after this chunk (a repeated maximum counts twice)
+        r.m2 = (cm1 > r.m1) ? fmaxf(fmaxf(r.m1, s2), r.m2) : fmaxf(r.m2, cm1);
+      }
+      if (cm1 > r.m1) {
+        if (r.m1 > -INFINITY) r.s *= ex2((r.m1 - cm1) * kLog2e);
+        r.m1 = cm1;
+        // first position of the new maximum among this thread's values (positions increase with e)
+        const int tbase = static_cast<int>(base) + static_cast<int>(threadIdx.x) * (16 / ESZ);
+        int best = INT_MAX;
+#pragma unroll
+        for (int e = PER - 1; e >= 0; --e) {
+          const int pos = tbase + (e / (16 / ESZ)) * kStreamThreads * (16 / ESZ) + (e % (16 / ESZ));
+          best = (f[e] == cm1) ? pos : best;
+        }
+        r.idx = best;
+      }
+      if (r.m1 > -INFINITY) {
+        const float mb = r.m1 * kLog2e;
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int e = 0; e < PER; e += 2) {
+          float t0, t1;
+          ffma2(t0, t1, f[e], f[e + 1], kLog2e, kLog2e, -mb, -mb);
+          fadd2_acc(sa[(e >> 1) & 3], sb[(e >> 1) & 3], ex2(t0), ex2(t1));
+        }
+        r.s += ((sa[0] + sb[0]) + (sa[1] + sb[1])) + ((sa[2] + sb[2]) + (sa[3] + sb[3]));
+      }
+      // the slot has been read and used: refill it with the chunk kStreamStages ahead
+      issue(slot);
+      slot = (slot + 1) % kStreamStages;
+      cs.off += kStageBytes;
+      if (cs.off >= cs.bytes) chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
+    }
+    // block partial of the segment: per-warp shuffles, then warp 0 merges the eight
+    Partial pw{r.m1, r.s, r.idx, r.m2};
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) pw = merge(pw, shfl_partial(pw, d));
+    if (lane == 0) wpart[warp] = pw;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      Partial q = wpart[0];
+      for (int w2 = 1; w2 < kStreamThreads / 32; ++w2) q = merge(q, wpart[w2]);
+      part[item] = q;
+    }
+    __syncthreads();
   }
+  cp_async_wait<0>();
 }
 
 // Rows whose length or alignment rules out 16-byte vectors: one element per
@@ -314,9 +423,25 @@ UnmaskPlan plan_unmask(int64_t vocab, ssm_dtype dtype, const void* logits) {
   UnmaskPlan p;
   p.vector = ((vocab * esz) % 16 == 0) && (logits == nullptr || ssm::aligned16(logits));
   // both plans cut a row into the same chunks, so the workspace does not depend on the plan
-  p.chunk = static_cast<int64_t>(ssm::kUnmaskThreads) * ssm::kUnroll * vec;
+  p.chunk = static_cast<int64_t>(ssm::kUnmaskThreads) * ssm::kUnroll * vec;  // 64 KB segments
   p.n_chunks = static_cast<int>((vocab + p.chunk - 1) / p.chunk);
   return p;
+}
+
+// The ring exceeds the default 48 KB of dynamic shared memory: opt in once per device
+// and kernel (one static flag per instantiation of this function, i.e. per kernel).
+template <auto kernel>
+bool stream_attr_set(size_t bytes) {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (done.load() & bit) return true;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes)) !=
+      cudaSuccess)
+    return false;
+  done.fetch_or(bit);
+  return true;
 }
 
 }  // namespace
@@ -351,22 +476,44 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));
+  const size_t stream_smem = ssm::kStreamStages * ssm::kStageBytes + 128;  // 96 KB: two CTAs per SM
+  const int64_t n_items = rows * plan.n_chunks;
+  const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 6 * ssm::num_sms()));
+  unsigned* err = ssm::device_error_word();
+  const uint64_t wait_ns = ssm::wait_limit_ns();
+  const bool need_second = p2 != nullptr || mode == SSM_COMMIT_MARGIN;
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
-    if (plan.vector)
-      ssm::unmask_partial_vec_kernel<__nv_bfloat16, ssm::kUnroll><<<grid, ssm::kUnmaskThreads, 0, st>>>(
-          x, vocab, plan.chunk, plan.n_chunks, masked, part);
-    else
+    if (plan.vector) {
+      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem) ||
+          !stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, false>>(stream_smem))
+        return SSM_ERR_CUDA;
+      if (need_second)
+        ssm::unmask_stream_kernel<__nv_bfloat16, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+      else
+        ssm::unmask_stream_kernel<__nv_bfloat16, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+    } else {
       ssm::unmask_partial_scalar_kernel<__nv_bfloat16><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
+    }
   } else {
     auto* x = static_cast<const float*>(logits);
-    if (plan.vector)
-      ssm::unmask_partial_vec_kernel<float, ssm::kUnroll><<<grid, ssm::kUnmaskThreads, 0, st>>>(
-          x, vocab, plan.chunk, plan.n_chunks, masked, part);
-    else
+    if (plan.vector) {
+      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem) ||
+          !stream_attr_set<ssm::unmask_stream_kernel<float, false>>(stream_smem))
+        return SSM_ERR_CUDA;
+      if (need_second)
+        ssm::unmask_stream_kernel<float, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+      else
+        ssm::unmask_stream_kernel<float, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+    } else {
       ssm::unmask_partial_scalar_kernel<float><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
+    }
   }
   ssm_status s = ssm::launch_status();
   if (s != SSM_OK) return s;
