@@ -12,11 +12,12 @@
 //    kv head, pair of 128-row query tiles), taken round-robin; barrier phases
 //    carry over from unit to unit, so the next unit's Q/K loads and first
 //    QK^T overlap the current unit's last softmax and epilogue.  Per unit,
-//    warp 0 streams K/V tiles with TMA (128 keys = four 32-row
-//    sub-boxes, so the cache segment and the new-row segment pack back to back
-//    with at most 31 padded keys each; 3-stage K ring, 2-stage V ring).  Warp 1
-//    issues tcgen05.mma: S = Q K^T from shared memory into tensor memory, and
-//    O += P V with P read from tensor memory.  Two softmax warpgroups ("slots"
+//    warps 0 and 2 stream the K and the V tiles with TMA, each ring at its own
+//    pace (128 keys = four 32-row sub-boxes, so the cache segment and the
+//    new-row segment pack back to back with at most 31 padded keys each;
+//    3-stage K ring, 2-stage V ring).  Warp 1 issues tcgen05.mma: S = Q K^T
+//    from shared memory into tensor memory, and O += P V with P read from
+//    tensor memory.  Two softmax warpgroups ("slots"
 //    A and B, one query row per thread) alternate: while one turns its S tile
 //    into P (written back over S as bf16), the tensor core runs the other
 //    slot's GEMMs.  With two query tiles each slot owns one; with a single
@@ -40,7 +41,15 @@ namespace {
 constexpr int kBM = 128;            // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;            // keys per tile (tcgen05 N of QK^T, K of PV)
 constexpr int kSub = 32;            // rows per TMA sub-box of a key tile
-constexpr int kAttnThreads = 320;   // warp 0: TMA, warp 1: MMA, warps 2-5: slot A, warps 6-9: slot B
+constexpr int kAttnThreads = 384;   // warpgroup 0: TMA Q/K (warp 0), MMA (warp 1), TMA V (warp 2); warpgroups 1, 2: slots A, B
+// Register split: the kernel is launched with kLaunchRegs per thread (checked on the host);
+// warpgroup 0 gives back down to kCtrlRegs and the two softmax warpgroups grow to
+// kSoftmaxRegs: 128 * (168 - 72) = 256 * (216 - 168), so the split adds up exactly.
+constexpr int kLaunchRegs = 168;
+constexpr int kCtrlRegs = 72;
+constexpr int kSoftmaxRegs = 216;
+static_assert(128 * (kLaunchRegs - kCtrlRegs) >= 256 * (kSoftmaxRegs - kLaunchRegs), "register split");
+static_assert(kAttnThreads * kLaunchRegs <= 65536, "launch registers");
 constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
 constexpr int kKStages = 3;
 constexpr int kVStages = 2;
@@ -323,43 +332,45 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
   tc_fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------- TMA producer
-    if (lane == 0) {
-      bool ok = true;
-      int qcount = 0;            // units whose Q was loaded
-      int kfill = 0, vfill = 0;  // K / V tiles loaded so far (all units)
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit w = make_unit(p, u);
-        if (!w.valid) continue;
-        if (qcount > 0) ok = mbar_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
-        if (!ok) break;
-        const int nq = w.two ? 2 : 1;
-        mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
-        for (int x = 0; x < nq; ++x) {
-          int qy, qz;
-          if (uniform) {
-            qy = (w.qt0 + x) * kBM;
-            qz = w.prob * p.h_kv + w.g;
-          } else {
-            qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
-                 (w.qt0 + x) * kBM;
-            qz = 0;
+  if (warp < 4) {
+    // warpgroup 0 gives registers back (all four warps, one instruction)
+    setmaxnreg_dec<kCtrlRegs>();
+    if (warp == 0 || warp == 2) {
+      // ------------------------------------------------------------- TMA producers
+      // warp 0 loads Q and the K ring, warp 2 the V ring, each at its own pace
+      const int half = warp == 2 ? 1 : 0;
+      if (lane == 0) {
+        bool ok = true;
+        int qcount = 0;  // units whose Q was loaded
+        int fills = 0;   // tiles loaded into this ring so far (all units)
+        const int nst = half ? kVStages : kKStages;
+        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+          const Unit w = make_unit(p, u);
+          if (!w.valid) continue;
+          if (!half) {
+            if (qcount > 0) ok = mbar_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
+            if (!ok) break;
+            const int nq = w.two ? 2 : 1;
+            mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
+            for (int x = 0; x < nq; ++x) {
+              int qy, qz;
+              if (uniform) {
+                qy = (w.qt0 + x) * kBM;
+                qz = w.prob * p.h_kv + w.g;
+              } else {
+                qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
+                     (w.qt0 + x) * kBM;
+                qz = 0;
+              }
+  #pragma unroll
+              for (int pn = 0; pn < NP; ++pn)
+                tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+            }
+            ++qcount;
           }
-#pragma unroll
-          for (int pn = 0; pn < NP; ++pn)
-            tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
-        }
-        ++qcount;
-        const int c3 = uniform ? w.prob : 0;
-        // K runs one tile ahead of V: K(j) then V(j - 1)
-        for (int j = 0; j <= w.nt && ok; ++j) {
-          for (int half = 0; half < 2 && ok; ++half) {
-            const int jt = half ? j - 1 : j;
-            if (jt < 0 || jt >= w.nt) continue;
-            const int nst = half ? kVStages : kKStages;
-            const int idx = half ? vfill : kfill;
-            const int st = idx % nst, fill = idx / nst;
+          const int c3 = uniform ? w.prob : 0;
+          for (int jt = 0; jt < w.nt && ok; ++jt) {
+            const int st = fills % nst, fill = fills / nst;
             if (fill > 0) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
             if (!ok) break;
             uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
@@ -373,10 +384,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
               const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
                                          : (uniform ? (sub0 - w.n_csub) * kSub
                                                     : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
-#pragma unroll
+  #pragma unroll
               for (int pn = 0; pn < NP; ++pn) tma_load_4d(dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
             } else
-#pragma unroll
+  #pragma unroll
             for (int sb = 0; sb < 4; ++sb) {
               const int sub = 4 * jt + sb;
               const CUtensorMap* map;
@@ -391,112 +402,110 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
                 map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
                 c2 = p.new_rows_extent;
               }
-#pragma unroll
+  #pragma unroll
               for (int pn = 0; pn < NP; ++pn)
                 tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
             }
-            if (half) ++vfill;
-            else ++kfill;
+            ++fills;
           }
         }
-      }
-      if (!ok) {
-        record_error(p.err, SSM_ERR_TIMEOUT);
-        // let every copy in flight land before the CTA's shared memory is released:
-        // the newest fill of each stage is the only one that can still be in flight
-        if (qcount > 0) mbar_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
-        for (int i = max(0, kfill - kKStages); i < kfill; ++i)
-          mbar_wait(&bars[K_FULL + i % kKStages], (i / kKStages) & 1, kDrainNs);
-        for (int i = max(0, vfill - kVStages); i < vfill; ++i)
-          mbar_wait(&bars[V_FULL + i % kVStages], (i / kVStages) & 1, kDrainNs);
-      }
-    }
-    __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      bool ok = true;
-      // operand descriptors: the per-instruction ones differ only in the start address field
-      const uint64_t dQ = sdesc_sw128(smem_u32(smem + L::Q), 16, 1024);
-      const uint64_t dK = sdesc_sw128(smem_u32(smem + L::K), 16, 1024);
-      const uint64_t dV = sdesc_sw128(smem_u32(smem + L::V), kPanel, 1024);
-      int ucount = 0;            // units processed
-      int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
-      int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit w = make_unit(p, u);
-        if (!w.valid) continue;
-        ok = mbar_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
-        if (!ok) break;
-        int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
-        int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
-        bool freed0 = false, freed1 = false;
-        // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O
-        auto wait_o_free = [&](int x) -> bool {
-          bool& f = x ? freed1 : freed0;
-          if (f) return true;
-          f = true;
-          return ucount == 0 || mbar_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
-        };
-        // O_X += P_X V(j) for slot X's latest job
-        auto issue_pv = [&](int x) -> bool {
-          const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
-          int& pv = x ? pv1 : pv0;
-          if (!wait_o_free(x)) return false;
-          if (!mbar_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
-          const int vi = vbase + jp;
-          if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
-          tc_fence_after_sync();
-          const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
-          const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
-          const uint32_t acc0 = k > 0 ? 1u : 0u;
-#pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk)
-            umma_bf16_ts(d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4), kIdescPV,
-                         kk > 0 ? 1u : acc0);
-          umma_commit(&bars[O_DONE + x]);
-          if (!w.two || x == 1) umma_commit(&bars[V_EMPTY + vi % kVStages]);
-          ++pv;
-          return true;
-        };
-        const int n_jobs = w.two ? 2 * w.nt : w.nt;
-        for (int t = 0; t < n_jobs && ok; ++t) {
-          const int x = t & 1;
-          const int j = w.two ? (t >> 1) : t;
-          if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
-          if (!ok) break;
-          const int ki = kbase + j;
-          ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
-          if (!ok) break;
-          const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
-          const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
-          const uint32_t s_tmem = tmem + x * kBN;
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
-            umma_bf16_ss(s_tmem, qb + off, kb + off, kIdescQK, kk > 0 ? 1u : 0u);
-          }
-          umma_commit(&bars[S_FULL + x]);
-          if (!w.two || x == 1) umma_commit(&bars[K_EMPTY + ki % kKStages]);
-          if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
+        if (!ok) {
+          record_error(p.err, SSM_ERR_TIMEOUT);
+          // let every copy in flight land before the CTA's shared memory is released:
+          // the newest fill of each stage is the only one that can still be in flight
+          if (!half && qcount > 0) mbar_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
+          for (int i = max(0, fills - nst); i < fills; ++i)
+            mbar_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
         }
-        if (ok) umma_commit(&bars[Q_EMPTY]);
-        if (ok && kx0 > 0) ok = issue_pv(0);
-        if (ok && kx1 > 0) ok = issue_pv(1);
-        if (ok) ok = wait_o_free(0) && wait_o_free(1);
-        kbase += w.nt;
-        vbase += w.nt;
-        ++ucount;
       }
-      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
-      // every issued MMA completes before tensor memory is released
-      umma_commit(&bars[DRAIN]);
-      mbar_wait(&bars[DRAIN], 0, kDrainNs);
+      __syncwarp();
+    } else if (warp == 1) {
+      // ------------------------------------------------------------- MMA issuer
+      if (lane == 0) {
+        bool ok = true;
+        // operand descriptors: the per-instruction ones differ only in the start address field
+        const uint64_t dQ = sdesc_sw128(smem_u32(smem + L::Q), 16, 1024);
+        const uint64_t dK = sdesc_sw128(smem_u32(smem + L::K), 16, 1024);
+        const uint64_t dV = sdesc_sw128(smem_u32(smem + L::V), kPanel, 1024);
+        int ucount = 0;            // units processed
+        int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
+        int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
+        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+          const Unit w = make_unit(p, u);
+          if (!w.valid) continue;
+          ok = mbar_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
+          if (!ok) break;
+          int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
+          int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
+          bool freed0 = false, freed1 = false;
+          // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O
+          auto wait_o_free = [&](int x) -> bool {
+            bool& f = x ? freed1 : freed0;
+            if (f) return true;
+            f = true;
+            return ucount == 0 || mbar_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
+          };
+          // O_X += P_X V(j) for slot X's latest job
+          auto issue_pv = [&](int x) -> bool {
+            const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
+            int& pv = x ? pv1 : pv0;
+            if (!wait_o_free(x)) return false;
+            if (!mbar_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
+            const int vi = vbase + jp;
+            if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
+            tc_fence_after_sync();
+            const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
+            const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
+            const uint32_t acc0 = k > 0 ? 1u : 0u;
+  #pragma unroll
+            for (int kk = 0; kk < kBN / 16; ++kk)
+              umma_bf16_ts(d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4), kIdescPV,
+                           kk > 0 ? 1u : acc0);
+            umma_commit(&bars[O_DONE + x]);
+            if (!w.two || x == 1) umma_commit(&bars[V_EMPTY + vi % kVStages]);
+            ++pv;
+            return true;
+          };
+          const int n_jobs = w.two ? 2 * w.nt : w.nt;
+          for (int t = 0; t < n_jobs && ok; ++t) {
+            const int x = t & 1;
+            const int j = w.two ? (t >> 1) : t;
+            if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
+            if (!ok) break;
+            const int ki = kbase + j;
+            ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
+            if (!ok) break;
+            const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
+            const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
+            const uint32_t s_tmem = tmem + x * kBN;
+  #pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
+              umma_bf16_ss(s_tmem, qb + off, kb + off, kIdescQK, kk > 0 ? 1u : 0u);
+            }
+            umma_commit(&bars[S_FULL + x]);
+            if (!w.two || x == 1) umma_commit(&bars[K_EMPTY + ki % kKStages]);
+            if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
+          }
+          if (ok) umma_commit(&bars[Q_EMPTY]);
+          if (ok && kx0 > 0) ok = issue_pv(0);
+          if (ok && kx1 > 0) ok = issue_pv(1);
+          if (ok) ok = wait_o_free(0) && wait_o_free(1);
+          kbase += w.nt;
+          vbase += w.nt;
+          ++ucount;
+        }
+        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+        // every issued MMA completes before tensor memory is released
+        umma_commit(&bars[DRAIN]);
+        mbar_wait(&bars[DRAIN], 0, kDrainNs);
+      }
+      __syncwarp();
     }
-    __syncwarp();
   } else {
-    // ------------------------------------------------------------- softmax slots (warps 2..9)
-    const int x = (warp - 2) >> 2;   // slot
+    // ------------------------------------------------------------- softmax slots (warps 4..11, warpgroups 1 and 2)
+    setmaxnreg_inc<kSoftmaxRegs>();
+    const int x = (warp - 4) >> 2;   // slot
     const int quarter = warp & 3;    // TMEM lanes 32*quarter .. +31 belong to this warp
     const int row = quarter * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
@@ -578,7 +587,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       if (ok && jobs > 0) ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
       if (!ok) break;
       tc_fence_after_sync();
-      // split keys: slot B hands its (max, sum) to slot A, which merges both accumulators
       // Split keys: slot B hands its (max, sum) to slot A, which merges both accumulators.
       // The buffer is rewritten only after slot B's last PV of a later unit, which the MMA
       // issues after slot A freed this unit's accumulators, i.e. after slot A's reads.
@@ -746,6 +754,18 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                                                           rope_theta, max_n_new, qhat, khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK) return s;
+  }
+  // the warpgroup register split assumes the compiled register count
+  {
+    static std::atomic<int> regs_ok{0};  // 0 unknown, 1 ok, 2 mismatch
+    int st_regs = regs_ok.load();
+    if (st_regs == 0) {
+      cudaFuncAttributes fa;
+      if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D>) != cudaSuccess) return SSM_ERR_CUDA;
+      st_regs = fa.numRegs == kLaunchRegs ? 1 : 2;
+      regs_ok.store(st_regs);
+    }
+    if (st_regs != 1) return SSM_ERR_UNSUPPORTED;
   }
   // the dynamic shared-memory opt-in is a per-device function attribute
   static std::atomic<uint64_t> attr_set{0};
