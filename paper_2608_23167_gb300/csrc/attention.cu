@@ -308,7 +308,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&bars[S_FULL + x], 1);
-      mbar_init(&bars[P_FULL + x], 4);   // one arrival per softmax warp
+      mbar_init(&bars[P_FULL + x], 5);   // one arrival per softmax warp, one from the K/V watcher
       mbar_init(&bars[O_DONE + x], 1);
       mbar_init(&bars[O_FREE + x], 4);
     }
@@ -450,9 +450,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
             const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
             int& pv = x ? pv1 : pv0;
             if (!wait_o_free(x)) return false;
+            // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
             if (!mbar_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
             const int vi = vbase + jp;
-            if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
             tc_fence_after_sync();
             const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
             const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
@@ -470,10 +470,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           for (int t = 0; t < n_jobs && ok; ++t) {
             const int x = t & 1;
             const int j = w.two ? (t >> 1) : t;
-            if ((x ? kx1 : kx0) > 0) ok = issue_pv(x);
-            if (!ok) break;
             const int ki = kbase + j;
-            ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
+            if ((x ? kx1 : kx0) > 0)
+              ok = issue_pv(x);
+            else
+              ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
             if (!ok) break;
             const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
             const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
@@ -499,6 +500,50 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         // every issued MMA completes before tensor memory is released
         umma_commit(&bars[DRAIN]);
         mbar_wait(&bars[DRAIN], 0, kDrainNs);
+      }
+      __syncwarp();
+    } else {
+      // ------------------------------------------------------------- K/V watcher (warp 3)
+      // Every mbarrier test costs the MMA-issuing thread ~150 cycles in which it
+      // issues nothing, so this warp takes the K and V waits off it: it walks the
+      // issuer's step order and, for each PV, waits until V of that PV and the K
+      // tile of the slot's next QK^T have landed, then adds its arrival to the
+      // slot's P_FULL phase.  The issuer then waits for P_FULL alone.  To land in
+      // the right phase it first waits for the slot's previous phase to complete.
+      if (lane == 0) {
+        bool ok = true;
+        int kbase = 0;
+        int done0 = 0, done1 = 0;  // P_FULL phases this warp has arrived on, per slot
+        // one arrival for slot x's PV of tile jp, whose slot next reads K tile jk (-1: none)
+        auto vouch = [&](int x, int jp, int jk) -> bool {
+          int& d = x ? done1 : done0;
+          if (d > 0 && !mbar_wait(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
+          const int vi = kbase + jp;
+          if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
+          if (jk >= 0) {
+            const int ki = kbase + jk;
+            if (!mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns)) return false;
+          }
+          mbar_arrive(&bars[P_FULL + x]);
+          ++d;
+          return true;
+        };
+        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+          const Unit w = make_unit(p, u);
+          if (!w.valid) continue;
+          int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
+          const int n_jobs = w.two ? 2 * w.nt : w.nt;
+          for (int t = 0; t < n_jobs && ok; ++t) {
+            const int x = t & 1;
+            const int j = w.two ? (t >> 1) : t;
+            if ((x ? kx1 : kx0) > 0) ok = vouch(x, x ? jlast1 : jlast0, j);
+            if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
+          }
+          if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
+          if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
+          kbase += w.nt;
+        }
+        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
       }
       __syncwarp();
     }
