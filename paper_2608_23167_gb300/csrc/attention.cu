@@ -17,13 +17,13 @@
 //    new-row segment pack back to back with at most 31 padded keys each;
 //    3-stage K ring, 2-stage V ring).  Warp 1 issues tcgen05.mma: S = Q K^T
 //    from shared memory into tensor memory, and O += P V with P read from
-//    tensor memory.  Two softmax warpgroups ("slots"
-//    A and B, one query row per thread) alternate: while one turns its S tile
-//    into P (written back over S as bf16), the tensor core runs the other
-//    slot's GEMMs.  With two query tiles each slot owns one; with a single
-//    query tile the slots split the key tiles (even/odd) and merge their
-//    partial softmax states at the end.  O is rescaled only when a row maximum
-//    grows by more than 2^8.
+//    tensor memory; warp 3 waits for the K and V tiles on its behalf.  Two
+//    softmax warpgroups ("slots" A and B, one query row per thread) alternate:
+//    while one turns its S tile into P (written back over S as bf16), the
+//    tensor core runs the other slot's GEMMs.  With two query tiles each slot
+//    owns one; with a single query tile the slots split the key tiles
+//    (even/odd) and merge their partial softmax states at the end.  O is
+//    rescaled only when a row maximum grows by more than 2^8.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
