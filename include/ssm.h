@@ -10,7 +10,7 @@
  *   3. ssm_attention          -- bidirectional MHA/GQA attention with rotary
  *                                encodings at the original positions
  *   4. ssm_unmask             -- vocabulary softmax, confidence, argmax and the
- *                                threshold / top-k / margin commit (Sec. 4.1, 4.5)
+ *                                threshold / top-k / margin commit (Sec. 4.2, 4.6)
  *
  * Conventions (all entry points):
  *   - Every function returns ssm_status; nothing throws across the ABI.
@@ -231,8 +231,8 @@ ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_
                                 ssm_stream_t stream);
 
 /* ------------------------------------------------------------------------- */
-/* 4. Confidence-based unmasking (Sec. 4.1 "Baselines": Vanilla top-1 and     */
-/*    parallel threshold decoding; Sec. 4.5: margin decoding).                */
+/* 4. Confidence-based unmasking (Sec. 4.2 "Baselines": Vanilla top-1 and     */
+/*    parallel threshold decoding; Sec. 4.6: margin decoding).                */
 /* ------------------------------------------------------------------------- */
 
 /* For every masked block position (masked[b, j] != 0): the softmax over the

@@ -17,8 +17,8 @@ in the paper's order:
                             encodings at the retained tokens' original positions
                             (Sec. 3.2, sparse input construction).
 * ``unmask``             -- parallel (threshold) decoding and Vanilla top-1
-                            decoding (Sec. 4.1 "Baselines"), and the margin rule
-                            (Sec. 4.5).
+                            decoding (Sec. 4.2 "Baselines"), and the margin rule
+                            (Sec. 4.6).
 * ``bf16_round``         -- round-to-nearest-even to bfloat16 (the storage type
                             of the sparse input).
 
@@ -313,11 +313,11 @@ def unmask(logits: np.ndarray, masked: np.ndarray, mode: int = MODE_THRESHOLD,
     """Which masked positions of the current block are decoded this step.
 
     logits: [batch, B, V]; masked: [batch, B] (nonzero = still [MASK]).
-    * threshold ("Par.", Sec. 4.1): commit every masked position whose
+    * threshold ("Par.", Sec. 4.2): commit every masked position whose
       confidence is above the threshold (read as strictly greater);
-    * top-k (Vanilla is k = 1, Sec. 4.1): commit the k masked positions of
+    * top-k (Vanilla is k = 1, Sec. 4.2): commit the k masked positions of
       highest confidence;
-    * margin (Sec. 4.5): commit masked positions whose top-1 minus top-2
+    * margin (Sec. 4.6): commit masked positions whose top-1 minus top-2
       probability is above the threshold.
     Reading (threshold and margin): when fewer than min_commit positions pass,
     the highest-confidence remaining masked positions are added, so that each

@@ -15,7 +15,7 @@
 //    warps 0 and 2 stream the K and the V tiles with TMA, each ring at its own
 //    pace (128 keys = four 32-row sub-boxes, so the cache segment and the
 //    new-row segment pack back to back with at most 31 padded keys each;
-//    3-stage K ring, 2-stage V ring).  Warp 1 issues tcgen05.mma: S = Q K^T
+//    2-stage K ring, 3-stage V ring).  Warp 1 issues tcgen05.mma: S = Q K^T
 //    from shared memory into tensor memory, and O += P V with P read from
 //    tensor memory; warp 3 waits for the K and V tiles on its behalf.  Two
 //    softmax warpgroups ("slots" A and B, one query row per thread) alternate:
@@ -51,8 +51,8 @@ constexpr int kSoftmaxRegs = 216;
 static_assert(128 * (kLaunchRegs - kCtrlRegs) >= 256 * (kSoftmaxRegs - kLaunchRegs), "register split");
 static_assert(kAttnThreads * kLaunchRegs <= 65536, "launch registers");
 constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
-constexpr int kKStages = 3;
-constexpr int kVStages = 2;
+constexpr int kKStages = 2;
+constexpr int kVStages = 3;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8

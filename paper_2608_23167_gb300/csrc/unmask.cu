@@ -1,5 +1,5 @@
-// unmask.cu -- confidence-based unmasking (Sec. 4.1 "Baselines": Vanilla top-1
-// and parallel threshold decoding; Sec. 4.5: margin decoding).
+// unmask.cu -- confidence-based unmasking (Sec. 4.2 "Baselines": Vanilla top-1
+// and parallel threshold decoding; Sec. 4.6: margin decoding).
 //
 // Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
 // segments of 32768 entries (the work items, dealt round-robin to persistent
