@@ -366,6 +366,42 @@ def oracle_sample(w: W.Workload, budget_s: float, seed: int = 99):
     return done / t_used, done, t_used, used
 
 
+def _event_ms(fn, reps: int, warmup: int = 3) -> float:
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def time_next_rows(w: W.Workload, dev, hbm_peak: float) -> dict:
+    """Secondary measurements of the rows that extend the step (not in the timed step).
+
+    cache_append: the prefix-cache update at block boundaries, 8192 rows of this workload's
+    K/V heads (one sequence; 268 MB moved, more than L2) appended into an 8192-row cache.
+    """
+    from paper_2608_23167_gb300 import ssm
+    out = {}
+    n = 8192
+    kn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 71).to(dev)
+    vn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 72).to(dev)
+    kc = torch.empty_like(kn)
+    vc = torch.empty_like(vn)
+    pos = torch.arange(n, dtype=torch.int32, device=dev)
+    ms = _event_ms(lambda: ssm.ssm_cache_append(kn, vn, pos, kc, vc, 0, w.rope_theta), reps=20)
+    nbytes = 4.0 * n * w.h_kv * w.head_dim * 2
+    out["cache_append"] = {"rows": n, "ms": ms, "GBps": nbytes / (ms * 1e-3) / 1e9,
+                           "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm_peak,
+                           "bytes": "K and V rows read once and written once (rotated K)"}
+    del kn, vn, kc, vc
+    return out
+
+
 def reduce_max(x: float, device, dist_on: bool) -> float:
     """Max over ranks of a per-rank time (the job ends when its slowest replica ends)."""
     if not dist_on:
@@ -432,6 +468,7 @@ def main():
     ap.add_argument("--workload", default="long", choices=list(W.WORKLOADS))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-next", action="store_true", help="skip the secondary measurements of the next rows")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -508,6 +545,12 @@ def main():
         "unmask_frac_8TBps_nominal": gb(inp.unmask_bytes(), unmask_ms) / 8000.0,
     }
 
+    next_rows = None
+    if rank == 0 and not args.no_next:
+        next_rows = time_next_rows(w, dev, hbm_peak)
+        if ssm.ssm_get_device_error() != 0:
+            raise RuntimeError("device error in the secondary measurements")
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         budget = float(os.environ.get("SSM_CPU_BASELINE_BUDGET_S", "15"))
@@ -527,6 +570,7 @@ def main():
                            (inp.gather_bytes() + inp.attn_bytes() + inp.unmask_bytes()) / 1e6)},
             "roofline": roofline, "stages": stages, "clocks": clk, "e2e": e2e,
             "cpu_baseline": cpu, "gpu_launches": StepInputs.LAUNCHES_PER_STEP * args.steps,
+            "next_rows": next_rows,
         }
         print(json.dumps(line), flush=True)
     if dist_on:

@@ -11,6 +11,8 @@
  *                                encodings at the original positions
  *   4. ssm_unmask             -- vocabulary softmax, confidence, argmax and the
  *                                threshold / top-k / margin commit (Sec. 4.2, 4.6)
+ * and, around the step, ssm_cache_append (the prefix-cache update at a block
+ * boundary, Sec. 4.8 "+PC.").
  *
  * Conventions (all entry points):
  *   - Every function returns ssm_status; nothing throws across the ABI.
@@ -286,6 +288,28 @@ ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, int32_t batch
                               int64_t vocab, const uint8_t* masked, ssm_commit_mode mode, float threshold,
                               int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
                               uint8_t* commit, ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 5. Prefix-cache append at a block boundary (prefix caching, "+PC." of      */
+/*    Sec. 4.8, Table 4).                                                      */
+/* ------------------------------------------------------------------------- */
+
+/* Once a block is decoded, the keys and values of its rows join the prefix
+ * cache that ssm_attention reads as already rotated: for every sequence b and
+ * row i < n_rows,
+ *   k_cache[b, start_row + i, h, :] = RoPE(k_new[b, i, h, :], pos[i], rope_theta)
+ *   v_cache[b, start_row + i, h, :] = v_new[b, i, h, :]
+ * with ssm_attention's rotation (the same bf16 bits as its pre-pass produces for
+ * the same key and position).  Other cache rows are not touched.
+ *   k_new, v_new      bf16 [batch, n_rows, h_kv, d]
+ *   pos               int32 [n_rows] (shared by the batch)
+ *   k_cache, v_cache  bf16 [batch, cache_rows, h_kv, d], caller-owned, written
+ *                     in place; they must not overlap k_new / v_new.
+ * d in {64, 128}; every bf16 pointer 16-byte aligned.  start_row + n_rows >
+ * cache_rows returns SSM_ERR_CAPACITY and writes nothing. */
+ssm_status ssm_cache_append(const void* k_new, const void* v_new, const int32_t* pos, int32_t batch,
+                            int32_t n_rows, int32_t h_kv, int32_t head_dim, float rope_theta, void* k_cache,
+                            void* v_cache, int64_t cache_rows, int64_t start_row, ssm_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -19,6 +19,10 @@ in the paper's order:
 * ``unmask``             -- parallel (threshold) decoding and Vanilla top-1
                             decoding (Sec. 4.2 "Baselines"), and the margin rule
                             (Sec. 4.6).
+* ``cache_append``       -- the prefix-cache update at a block boundary in the
+                            prefix-caching setting ("+PC.", Sec. 4.8, Table 4):
+                            the block's keys (rotated at their positions) and
+                            values are written into the cache.
 * ``bf16_round``         -- round-to-nearest-even to bfloat16 (the storage type
                             of the sparse input).
 
@@ -280,6 +284,27 @@ def attention(q: np.ndarray, k_new: np.ndarray, v_new: np.ndarray, pos: np.ndarr
             out[bi, :, h, :] = (p @ vals[bi, :, g, :]) / l
             lse[bi, :, h] = (m + np.log(l))[:, 0]
     return out, lse
+
+
+def cache_append(k_cache: np.ndarray, v_cache: np.ndarray, k_new: np.ndarray, v_new: np.ndarray,
+                 pos: np.ndarray, theta: float, start_row: int):
+    """Prefix-cache append at a block boundary (prefix caching, Sec. 4.8 "+PC.").
+
+    k_cache, v_cache: [batch, cache_rows, Hkv, d]; k_new, v_new: [batch, n, Hkv, d];
+    pos: [n] original positions of the new rows (shared by the batch).
+    Returns new (k_cache, v_cache) in float64 where rows start_row .. start_row+n-1
+    hold rope(k_new, pos) and v_new, and every other row is unchanged.  Reading:
+    the cache stores keys already rotated at their own positions, which is how
+    ``attention`` consumes it.  Raises ValueError when the rows do not fit.
+    """
+    k_cache = np.array(k_cache, dtype=np.float64)
+    v_cache = np.array(v_cache, dtype=np.float64)
+    n = k_new.shape[1]
+    if start_row < 0 or start_row + n > k_cache.shape[1]:
+        raise ValueError("appended rows do not fit in the cache")
+    k_cache[:, start_row:start_row + n] = rope(np.asarray(k_new, dtype=np.float64), pos, theta)
+    v_cache[:, start_row:start_row + n] = np.asarray(v_new, dtype=np.float64)
+    return k_cache, v_cache
 
 
 # --------------------------------------------------------------------------------------

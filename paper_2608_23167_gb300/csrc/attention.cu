@@ -32,6 +32,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "rope.cuh"
 #include "sm100_ptx.cuh"
 #include "tmem_io.cuh"
 
@@ -139,9 +140,8 @@ constexpr int kRopeWarps = 8;
 
 // One warp per new row.  Each lane owns four rotation pairs (i, i + D/2) of one
 // head vector, so D/8 lanes cover a head and a warp moves 32/(D/8) heads per
-// pass with 8-byte loads and stores.  The angles pos * theta^(-2i/D) are formed
-// and reduced modulo 2*pi in fp64 (inverse frequencies once per CTA), then
-// sin/cos are taken in fp32 on the reduced angle.
+// pass with 8-byte loads and stores.  The rotation is rope.cuh's (inverse
+// frequencies once per CTA).
 template <int D>
 __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
@@ -150,8 +150,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
   constexpr int LPH = D / 8;        // lanes per head vector
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
-  if (threadIdx.x < D / 2)
-    inv_freq[threadIdx.x] = theta > 0.f ? exp2(-(2.0 * threadIdx.x / D) * log2(static_cast<double>(theta))) : 0.0;
+  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane % LPH;       // which 4 pairs
@@ -163,13 +162,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
   const int32_t ps = pos[p.problems ? gm.new_row + i : i];
   float cs[4], sn[4];
 #pragma unroll
-  for (int t = 0; t < 4; ++t) {
-    const double a = static_cast<double>(ps) * inv_freq[4 * sub + t];
-    const double kk = rint(a * 0.15915494309189535);               // a / (2 pi)
-    double r = fma(-kk, 6.283185307179586, a);                      // 2 pi, high part
-    r = fma(-kk, 2.4492935982947064e-16, r);                        // 2 pi, low part
-    sincosf(static_cast<float>(r), &sn[t], &cs[t]);
-  }
+  for (int t = 0; t < 4; ++t) rope_sincos(ps, inv_freq[4 * sub + t], sn[t], cs[t]);
   const int64_t row = gm.new_row + i;
   const int n_vec = p.h_q + p.h_kv;
   for (int base = 0; base < n_vec; base += HPP * 4) {
@@ -188,16 +181,8 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       if (hv[u] >= n_vec) continue;
-      const float a[4] = {__uint_as_float(x1[u].x << 16), __uint_as_float(x1[u].x & 0xFFFF0000u),
-                          __uint_as_float(x1[u].y << 16), __uint_as_float(x1[u].y & 0xFFFF0000u)};
-      const float b[4] = {__uint_as_float(x2[u].x << 16), __uint_as_float(x2[u].x & 0xFFFF0000u),
-                          __uint_as_float(x2[u].y << 16), __uint_as_float(x2[u].y & 0xFFFF0000u)};
-      float y1[4], y2[4];
-#pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        y1[t] = a[t] * cs[t] - b[t] * sn[t];
-        y2[t] = b[t] * cs[t] + a[t] * sn[t];
-      }
+      uint2 y1, y2;
+      rope_rotate4(x1[u], x2[u], cs, sn, y1, y2);
       __nv_bfloat16* dst;
       if (hv[u] < p.h_q) {
         const int g = hv[u] / p.grp, hl = hv[u] - g * p.grp;
@@ -207,9 +192,8 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
       } else {
         dst = khat + (row * p.h_kv + (hv[u] - p.h_q)) * D;
       }
-      *reinterpret_cast<uint2*>(dst + 4 * sub) = make_uint2(pack_bf16x2(y1[0], y1[1]), pack_bf16x2(y1[2], y1[3]));
-      *reinterpret_cast<uint2*>(dst + D / 2 + 4 * sub) =
-          make_uint2(pack_bf16x2(y2[0], y2[1]), pack_bf16x2(y2[2], y2[3]));
+      *reinterpret_cast<uint2*>(dst + 4 * sub) = y1;
+      *reinterpret_cast<uint2*>(dst + D / 2 + 4 * sub) = y2;
     }
   }
 }

@@ -25,6 +25,8 @@ SSM_COMMIT_MARGIN = 2
 
 STATUS = {0: "ok", 1: "invalid argument", 2: "inconsistent shapes", 3: "capacity", 4: "CUDA error",
           5: "device wait timed out", 6: "unsupported", 7: "device input out of range"}
+SSM_OK, SSM_ERR_INVALID_ARG, SSM_ERR_SHAPE, SSM_ERR_CAPACITY = 0, 1, 2, 3
+SSM_ERR_CUDA, SSM_ERR_TIMEOUT, SSM_ERR_UNSUPPORTED, SSM_ERR_DEVICE_INPUT = 4, 5, 6, 7
 
 
 class SSMError(RuntimeError):
@@ -80,6 +82,7 @@ def lib() -> ctypes.CDLL:
                                           vp, vp, vp, vp, vp, sz, vp]),
             "ssm_unmask_noalloc": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32,
                                                   i32, vp, vp, vp, vp, vp]),
+            "ssm_cache_append": (ctypes.c_int, [vp, vp, vp, i32, i32, i32, i32, f32, vp, vp, i64, i64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -93,7 +96,8 @@ def exported_symbols() -> Sequence[str]:
     return ["ssm_status_str", "ssm_version", "ssm_get_device_error", "ssm_set_wait_limit_ns",
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
-            "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc"]
+            "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
+            "ssm_cache_append"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -250,6 +254,18 @@ def ssm_attention_varlen(q, k_new, v_new, pos, k_cache, v_cache, problems, n_pro
         _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(pos), _ptr(k_cache), _ptr(v_cache), total_new, total_cache,
         _ptr(problems), n_problems, max_n_new, max_n_cache, h_q, h_kv, d, float(rope_theta), float(scale),
         _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+# ------------------------------------------------------------------------------ prefix-cache append
+
+
+def ssm_cache_append(k_new, v_new, pos, k_cache, v_cache, start_row: int, rope_theta: float, stream=None):
+    """k_new, v_new: bf16 [batch, n_rows, h_kv, d]; k_cache, v_cache: bf16 [batch, cache_rows, h_kv, d],
+    written in place at rows start_row .. start_row + n_rows - 1."""
+    batch, n_rows, h_kv, d = k_new.shape
+    _check("ssm_cache_append", lib().ssm_cache_append(
+        _ptr(k_new), _ptr(v_new), _ptr(pos), batch, n_rows, h_kv, d, float(rope_theta), _ptr(k_cache),
+        _ptr(v_cache), k_cache.shape[1], int(start_row), _stream(stream)))
 
 
 # ------------------------------------------------------------------------------ unmask

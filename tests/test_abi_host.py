@@ -80,6 +80,11 @@ def test_argument_validation_without_device(lib):
                                     fake, None, None) == 1
     assert lib.ssm_build_step_input(fake, None, 1, 0, 32, 0, fake, 4, fake, 100, 60, 99, fake, fake, 5, 0.4,
                                     fake, None, None) == 6
+    # cache append: rows past the cache end, unsupported head_dim, negative start; zero rows is a no-op
+    assert lib.ssm_cache_append(fake, fake, fake, 1, 32, 4, 128, 1e4, fake, fake, 64, 40, None) == 3
+    assert lib.ssm_cache_append(fake, fake, fake, 1, 32, 4, 96, 1e4, fake, fake, 64, 0, None) == 6
+    assert lib.ssm_cache_append(fake, fake, fake, 1, 32, 4, 128, 1e4, fake, fake, 64, -1, None) == 1
+    assert lib.ssm_cache_append(None, None, None, 1, 0, 4, 128, 1e4, None, None, 64, 64, None) == 0
 
 
 def test_workspace_sizes(lib):

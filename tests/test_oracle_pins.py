@@ -286,6 +286,50 @@ def test_rope_relative_position():
         assert abs(a - b) < 1e-10
 
 
+# ----------------------------------------------------------------------------- prefix-cache append
+
+
+def test_cache_append_places_rotated_rows_and_leaves_the_rest():
+    # d = 2: one pair with inverse frequency 1, so a key at position p turns by p radians
+    rng = np.random.default_rng(21)
+    B, C, n, H = 2, 9, 3, 2
+    kc = rng.standard_normal((B, C, H, 2))
+    vc = rng.standard_normal((B, C, H, 2))
+    kn = rng.standard_normal((B, n, H, 2))
+    vn = rng.standard_normal((B, n, H, 2))
+    pos = np.array([40, 3, 1000])          # positions need not follow the row order
+    k2, v2 = O.cache_append(kc, vc, kn, vn, pos, 5e5, 4)
+    c, s_ = np.cos(pos)[None, :, None], np.sin(pos)[None, :, None]
+    want0 = kn[..., 0] * c - kn[..., 1] * s_
+    want1 = kn[..., 1] * c + kn[..., 0] * s_
+    assert np.allclose(k2[:, 4:7, :, 0], want0, atol=1e-12) and np.allclose(k2[:, 4:7, :, 1], want1, atol=1e-12)
+    assert np.array_equal(v2[:, 4:7], vn)
+    keep = np.r_[0:4, 7:9]
+    assert np.array_equal(k2[:, keep], kc[:, keep]) and np.array_equal(v2[:, keep], vc[:, keep])
+    # the inputs are not modified
+    assert not np.shares_memory(k2, kc)
+
+
+def test_cache_append_rotation_invariants_and_capacity():
+    rng = np.random.default_rng(22)
+    kn = rng.standard_normal((1, 6, 4, 64))
+    vn = rng.standard_normal((1, 6, 4, 64))
+    pos = np.arange(6) + 1024
+    kc, vc = O.cache_append(np.zeros((1, 16, 4, 64)), np.zeros((1, 16, 4, 64)), kn, vn, pos, 5e5, 10)
+    # a rotation keeps every head vector's norm
+    assert np.allclose(np.linalg.norm(kc[:, 10:], axis=-1), np.linalg.norm(kn, axis=-1))
+    # scores between two appended keys depend only on their position difference
+    kd, _ = O.cache_append(np.zeros((1, 16, 4, 64)), np.zeros((1, 16, 4, 64)), kn, vn, pos + 777, 5e5, 10)
+    g1 = np.einsum("nhd,mhd->hnm", kc[0, 10:], kc[0, 10:])
+    g2 = np.einsum("nhd,mhd->hnm", kd[0, 10:], kd[0, 10:])
+    assert np.allclose(g1, g2, atol=1e-9)
+    # theta == 0: no rotation, a plain copy
+    k0, _ = O.cache_append(np.zeros((1, 6, 4, 64)), np.zeros((1, 6, 4, 64)), kn, vn, pos, 0.0, 0)
+    assert np.array_equal(k0, kn)
+    with pytest.raises(ValueError):
+        O.cache_append(np.zeros((1, 16, 4, 64)), np.zeros((1, 16, 4, 64)), kn, vn, pos, 5e5, 11)
+
+
 def _attn_bruteforce(q, keys, vals, scale):
     out = []
     for qi in q:
