@@ -4,11 +4,15 @@
 // rows' positions, as every cached key is; Sec. 3.2 "Sparse Input
 // Construction": tokens keep their original positions).
 //
-// cache_append_kernel: one warp per (sequence, row).  A lane owns four
-// rotation pairs of one head vector (D/8 lanes per head, 8-byte accesses), the
-// rotation is rope.cuh's, so a key appended here carries the same bf16 bits as
-// the same key rotated by the attention's pre-pass.  Values are copied.
+// cache_append_kernel: persistent warps, one (sequence, row) at a time.  The
+// row's D/2 angles are formed once (two per lane) and shared through shared
+// memory; a lane then owns eight rotation pairs of one head vector (D/16 lanes
+// per head, 16-byte accesses, two head passes in flight).  The rotation is
+// rope.cuh's, so a key appended here carries the same bf16 bits as the same key
+// rotated by the attention's pre-pass.  Values are copied.
 #include <cuda_bf16.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "rope.cuh"
@@ -21,39 +25,69 @@ constexpr int kAppendWarps = 8;
 template <int D>
 __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
     const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
-    const int32_t* __restrict__ pos, int32_t n_rows, int32_t h_kv, float theta,
+    const int32_t* __restrict__ pos, int32_t batch, int32_t n_rows, int32_t h_kv, float theta,
     __nv_bfloat16* __restrict__ k_cache, __nv_bfloat16* __restrict__ v_cache, int64_t cache_rows,
     int64_t start_row) {
-  constexpr int LPH = D / 8;     // lanes per head vector
+  constexpr int LPH = D / 16;    // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;  // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
+  __shared__ float s_cs[kAppendWarps][D / 2], s_sn[kAppendWarps][D / 2];
   if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane % LPH, hoff = lane / LPH;
-  const int64_t b = blockIdx.y;
-  const int i = blockIdx.x * kAppendWarps + warp;
-  if (i >= n_rows) return;
-  float cs[4], sn[4];
+  const int64_t total = static_cast<int64_t>(batch) * n_rows;
+  // persistent warps over (sequence, row): the CTA's table is made once
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * kAppendWarps + warp; r < total;
+       r += static_cast<int64_t>(gridDim.x) * kAppendWarps) {
+    const int64_t b = r / n_rows;
+    const int i = static_cast<int>(r - b * n_rows);
+    // each pair's angle once per row (a lane takes pairs lane, lane + 32), shared through shared memory
+    const int32_t ps = pos[i];
+    __syncwarp();
 #pragma unroll
-  for (int t = 0; t < 4; ++t) rope_sincos(pos[i], inv_freq[4 * sub + t], sn[t], cs[t]);
-  const int64_t src_row = b * n_rows + i;
-  const int64_t dst_row = b * cache_rows + start_row + i;
-  for (int h = hoff; h < h_kv; h += HPP) {
-    const __nv_bfloat16* ks = k_new + (src_row * h_kv + h) * D;
-    const __nv_bfloat16* vs = v_new + (src_row * h_kv + h) * D;
-    __nv_bfloat16* kd = k_cache + (dst_row * h_kv + h) * D;
-    __nv_bfloat16* vd = v_cache + (dst_row * h_kv + h) * D;
-    const uint2 x1 = *reinterpret_cast<const uint2*>(ks + 4 * sub);
-    const uint2 x2 = *reinterpret_cast<const uint2*>(ks + D / 2 + 4 * sub);
-    const uint2 v1 = *reinterpret_cast<const uint2*>(vs + 4 * sub);
-    const uint2 v2 = *reinterpret_cast<const uint2*>(vs + D / 2 + 4 * sub);
-    uint2 y1, y2;
-    rope_rotate4(x1, x2, cs, sn, y1, y2);
-    *reinterpret_cast<uint2*>(kd + 4 * sub) = y1;
-    *reinterpret_cast<uint2*>(kd + D / 2 + 4 * sub) = y2;
-    *reinterpret_cast<uint2*>(vd + 4 * sub) = v1;
-    *reinterpret_cast<uint2*>(vd + D / 2 + 4 * sub) = v2;
+    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, inv_freq[t], s_sn[warp][t], s_cs[warp][t]);
+    __syncwarp();
+    float cs0[4], cs1[4], sn0[4], sn1[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      cs0[t] = s_cs[warp][8 * sub + t];
+      cs1[t] = s_cs[warp][8 * sub + 4 + t];
+      sn0[t] = s_sn[warp][8 * sub + t];
+      sn1[t] = s_sn[warp][8 * sub + 4 + t];
+    }
+    const int64_t src_row = r;
+    const int64_t dst_row = b * cache_rows + start_row + i;
+    // two head passes per iteration: eight 16-byte loads in flight per lane
+    for (int h0 = hoff; h0 < h_kv; h0 += 2 * HPP) {
+      uint4 x1[2], x2[2], v1[2], v2[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int h = h0 + u * HPP;
+        if (h < h_kv) {
+          const __nv_bfloat16* ks = k_new + (src_row * h_kv + h) * D + 8 * sub;
+          const __nv_bfloat16* vs = v_new + (src_row * h_kv + h) * D + 8 * sub;
+          x1[u] = *reinterpret_cast<const uint4*>(ks);
+          x2[u] = *reinterpret_cast<const uint4*>(ks + D / 2);
+          v1[u] = *reinterpret_cast<const uint4*>(vs);
+          v2[u] = *reinterpret_cast<const uint4*>(vs + D / 2);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int h = h0 + u * HPP;
+        if (h >= h_kv) continue;
+        uint2 ya, yb, yc, yd;
+        rope_rotate4(make_uint2(x1[u].x, x1[u].y), make_uint2(x2[u].x, x2[u].y), cs0, sn0, ya, yb);
+        rope_rotate4(make_uint2(x1[u].z, x1[u].w), make_uint2(x2[u].z, x2[u].w), cs1, sn1, yc, yd);
+        __nv_bfloat16* kd = k_cache + (dst_row * h_kv + h) * D + 8 * sub;
+        __nv_bfloat16* vd = v_cache + (dst_row * h_kv + h) * D + 8 * sub;
+        *reinterpret_cast<uint4*>(kd) = make_uint4(ya.x, ya.y, yc.x, yc.y);
+        *reinterpret_cast<uint4*>(kd + D / 2) = make_uint4(yb.x, yb.y, yd.x, yd.y);
+        *reinterpret_cast<uint4*>(vd) = v1[u];
+        *reinterpret_cast<uint4*>(vd + D / 2) = v2[u];
+      }
+    }
   }
 }
 
@@ -73,18 +107,18 @@ ssm_status ssm_cache_append(const void* k_new, const void* v_new, const int32_t*
   if (!k_new || !v_new || !pos || !k_cache || !v_cache) return SSM_ERR_INVALID_ARG;
   if (!ssm::aligned16(k_new) || !ssm::aligned16(v_new) || !ssm::aligned16(k_cache) || !ssm::aligned16(v_cache))
     return SSM_ERR_INVALID_ARG;
-  if (batch > 65535) return SSM_ERR_UNSUPPORTED;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid((n_rows + ssm::kAppendWarps - 1) / ssm::kAppendWarps, batch);
+  const int64_t warps_needed = (static_cast<int64_t>(batch) * n_rows + ssm::kAppendWarps - 1) / ssm::kAppendWarps;
+  const int grid = static_cast<int>(std::min<int64_t>(warps_needed, 8ll * ssm::num_sms()));
   const auto* kn = static_cast<const __nv_bfloat16*>(k_new);
   const auto* vn = static_cast<const __nv_bfloat16*>(v_new);
   auto* kc = static_cast<__nv_bfloat16*>(k_cache);
   auto* vc = static_cast<__nv_bfloat16*>(v_cache);
   if (head_dim == 128)
-    ssm::cache_append_kernel<128><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, n_rows, h_kv, rope_theta,
+    ssm::cache_append_kernel<128><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, batch, n_rows, h_kv, rope_theta,
                                                                          kc, vc, cache_rows, start_row);
   else
-    ssm::cache_append_kernel<64><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, n_rows, h_kv, rope_theta,
+    ssm::cache_append_kernel<64><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, batch, n_rows, h_kv, rope_theta,
                                                                         kc, vc, cache_rows, start_row);
   return ssm::launch_status();
 }
