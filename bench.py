@@ -379,14 +379,26 @@ def _event_ms(fn, reps: int, warmup: int = 3) -> float:
     return e0.elapsed_time(e1) / reps
 
 
-def time_next_rows(w: W.Workload, dev, hbm_peak: float) -> dict:
+def time_next_rows(w: W.Workload, n_suffix_rows: int, dev, hbm_peak: float) -> dict:
     """Secondary measurements of the rows that extend the step (not in the timed step).
 
+    suffix_topk: the next step's top-k candidates of every retained suffix position of one bench
+    step (this workload's vocabulary, bf16 N(0, sigma) stand-in logits, read once).
     cache_append: the prefix-cache update at block boundaries, 8192 rows of this workload's
     K/V heads (one sequence; 268 MB moved, more than L2) appended into an 8192-row cache.
     """
     from paper_2608_23167_gb300 import ssm
     out = {}
+    n = max(n_suffix_rows, 1)
+    lg = W.draw_logits((n, w.vocab), "bf16", w.logits_sigma, 73, device=dev)
+    ids = torch.empty((n, w.topk), dtype=torch.int32, device=dev)
+    pr = torch.empty((n, w.topk), dtype=torch.float32, device=dev)
+    ms = _event_ms(lambda: ssm.ssm_suffix_topk(lg, w.topk, ids, pr), reps=10)
+    nbytes = float(n) * w.vocab * 2
+    out["suffix_topk"] = {"rows": n, "k": w.topk, "ms": ms, "GBps": nbytes / (ms * 1e-3) / 1e9,
+                          "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm_peak,
+                          "bytes": "the logits of the retained suffix rows, read once"}
+    del lg, ids, pr
     n = 8192
     kn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 71).to(dev)
     vn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 72).to(dev)
@@ -547,7 +559,7 @@ def main():
 
     next_rows = None
     if rank == 0 and not args.no_next:
-        next_rows = time_next_rows(w, dev, hbm_peak)
+        next_rows = time_next_rows(w, inp.total_suffix, dev, hbm_peak)
         if ssm.ssm_get_device_error() != 0:
             raise RuntimeError("device error in the secondary measurements")
 

@@ -11,8 +11,9 @@
  *                                encodings at the original positions
  *   4. ssm_unmask             -- vocabulary softmax, confidence, argmax and the
  *                                threshold / top-k / margin commit (Sec. 4.2, 4.6)
- * and, around the step, ssm_cache_append (the prefix-cache update at a block
- * boundary, Sec. 4.8 "+PC.").
+ * and, around the step, ssm_suffix_topk (the retained suffix positions' top-k
+ * candidates for the next step's Eq. 6) and ssm_cache_append (the prefix-cache
+ * update at a block boundary, Sec. 4.8 "+PC.").
  *
  * Conventions (all entry points):
  *   - Every function returns ssm_status; nothing throws across the ABI.
@@ -288,6 +289,25 @@ ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, int32_t batch
                               int64_t vocab, const uint8_t* masked, ssm_commit_mode mode, float threshold,
                               int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
                               uint8_t* commit, ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 4b. The next step's soft-embedding candidates of the retained suffix       */
+/*     positions (Sec. 3.2 "Soft Suffix Embedding Mixing", the set T^i_{t+1}  */
+/*     and p^i_{t+1}(v) of Eq. 6).                                            */
+/* ------------------------------------------------------------------------- */
+
+/* For every row r of logits (one retained suffix position): ids[r, j] = the
+ * j-th most probable token (j < k; equal logits: lower id first) and
+ * probs[r, j] its probability under the softmax over the whole vocabulary
+ * (fp32; Eq. 6 renormalizes them within the set at the next step, which is
+ * what ssm_build_step_input's prev_topk_ids / prev_topk_prob take).
+ *   logits     bf16 or fp32 [n_rows, vocab], rows 16-byte aligned (vocab *
+ *              element size a multiple of 16 and logits 16-byte aligned;
+ *              otherwise SSM_ERR_UNSUPPORTED)
+ *   ids        int32 [n_rows, k];  probs  fp32 [n_rows, k]
+ * 1 <= k <= 8 (SSM_ERR_UNSUPPORTED otherwise), k <= vocab.  No workspace. */
+ssm_status ssm_suffix_topk(const void* logits, ssm_dtype dtype, int64_t n_rows, int64_t vocab, int32_t k,
+                           int32_t* ids, float* probs, ssm_stream_t stream);
 
 /* ------------------------------------------------------------------------- */
 /* 5. Prefix-cache append at a block boundary (prefix caching, "+PC." of      */

@@ -19,6 +19,11 @@ in the paper's order:
 * ``unmask``             -- parallel (threshold) decoding and Vanilla top-1
                             decoding (Sec. 4.2 "Baselines"), and the margin rule
                             (Sec. 4.6).
+* ``suffix_topk``        -- the top-k candidates of a retained suffix position
+                            and their probabilities under the full-vocabulary
+                            softmax (Sec. 3.2 "Soft Suffix Embedding Mixing": the
+                            set T^i_{t+1} and p^i_{t+1}(v) that Eq. 6 renormalizes
+                            at the next step).
 * ``cache_append``       -- the prefix-cache update at a block boundary in the
                             prefix-caching setting ("+PC.", Sec. 4.8, Table 4):
                             the block's keys (rotated at their positions) and
@@ -331,6 +336,32 @@ def token_confidence(logits_row: np.ndarray):
     p2 = float(order[-2]) if p.size > 1 else 0.0
     argmax = int(np.flatnonzero(l == m)[0])
     return conf, argmax, p2
+
+
+def suffix_topk(logits: np.ndarray, k: int):
+    """Top-k tokens of each row of logits [n, V] with their softmax probabilities.
+
+    Sec. 3.2 "Soft Suffix Embedding Mixing": for a retained suffix position the
+    next step takes the k most probable tokens under the current prediction
+    p(v) = softmax(logits)(v) and their probabilities (which Eq. 6 then
+    renormalizes within the set).  Returns ids int64 [n, k] in decreasing
+    probability and probs float64 [n, k] (full-vocabulary probabilities).
+    Readings: ties are broken by the lower token id; k > V is an error.
+    """
+    l = np.asarray(logits, dtype=np.float64)
+    n, V = l.shape
+    if not 1 <= k <= V:
+        raise ValueError("k must be in [1, V]")
+    ids = np.zeros((n, k), dtype=np.int64)
+    probs = np.zeros((n, k), dtype=np.float64)
+    for r in range(n):
+        m = l[r].max()
+        e = np.exp(l[r] - m)
+        p = e / e.sum()
+        order = np.lexsort((np.arange(V), -l[r]))[:k]      # by decreasing logit, then by id
+        ids[r] = order
+        probs[r] = p[order]
+    return ids, probs
 
 
 def unmask(logits: np.ndarray, masked: np.ndarray, mode: int = MODE_THRESHOLD,

@@ -45,10 +45,6 @@ __host__ __device__ inline SuffixGeom make_geom(const ssm_suffix_cfg& c) {
   return g;
 }
 
-__host__ __device__ inline int32_t tail_count(const SuffixGeom& g) {
-  return g.T >= g.B ? g.B : g.T;
-}
-
 // Is tail-block offset `o` one of the T evenly spaced offsets (j*(B-1))/(T-1)?
 __host__ __device__ inline bool tail_keeps(const SuffixGeom& g, int64_t o) {
   if (g.T <= 0) return false;

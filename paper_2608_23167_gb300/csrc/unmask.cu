@@ -23,6 +23,7 @@
 
 #include "common.cuh"
 #include "sm100_ptx.cuh"
+#include "stream.cuh"
 
 namespace ssm {
 namespace {
@@ -88,7 +89,6 @@ template <typename T>
 struct Vec;
 template <>
 struct Vec<__nv_bfloat16> {
-  static constexpr int N = 8;
   __device__ static void unpack(const uint4& v, float (&f)[8]) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
@@ -101,7 +101,6 @@ struct Vec<__nv_bfloat16> {
 };
 template <>
 struct Vec<float> {
-  static constexpr int N = 4;
   __device__ static void unpack(const uint4& v, float (&f)[4]) {
     f[0] = __uint_as_float(v.x);
     f[1] = __uint_as_float(v.y);
@@ -120,60 +119,12 @@ constexpr int kStageBytes = 16384;                     // one stage: 64 bytes pe
 constexpr int kStreamStages = 2;                       // chunks in flight per thread
 constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
 
-__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
-  uint32_t r;
-  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
-  return r;
-}
-__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
-  uint32_t r;
-  asm("min.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
-  return r;
-}
-__device__ __forceinline__ float lo_bf16(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float hi_bf16(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-
-// 16-byte asynchronous global -> shared copy (L2 only, bypassing L1).
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// Walks the chunks of this CTA's work items (masked rows only) in order.
-struct ChunkIter {
-  int64_t item, off, bytes, e0, row;
-  bool valid;
-};
-
 // Running per-thread state over one segment: max m1 (first index idx), second
 // largest m2 (a repeated maximum counts twice) and s = sum exp(x - m1).
 struct RunState {
   float m1, m2, s;
   int idx;
 };
-
-template <typename T>
-__device__ __forceinline__ void chunk_seek(ChunkIter& it, int64_t vocab, int64_t seg_elems, int n_seg,
-                                           int64_t n_items, const uint8_t* __restrict__ masked) {
-  // advance to the next item that has a masked row, if the current one is exhausted
-  while (it.item < n_items && (it.off >= it.bytes)) {
-    it.item += gridDim.x;
-    it.off = 0;
-    if (it.item >= n_items) break;
-    it.row = it.item / n_seg;
-    if (!masked[it.row]) {
-      it.bytes = 0;
-      continue;
-    }
-    it.e0 = (it.item - it.row * n_seg) * seg_elems;
-    it.bytes = (min(vocab, it.e0 + seg_elems) - it.e0) * static_cast<int64_t>(sizeof(T));
-  }
-  it.valid = it.item < n_items;
-}
 
 template <typename T, bool NEED_SECOND>
 __global__ void __launch_bounds__(kStreamThreads) unmask_stream_kernel(

@@ -83,6 +83,7 @@ def lib() -> ctypes.CDLL:
             "ssm_unmask_noalloc": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32,
                                                   i32, vp, vp, vp, vp, vp]),
             "ssm_cache_append": (ctypes.c_int, [vp, vp, vp, i32, i32, i32, i32, f32, vp, vp, i64, i64, vp]),
+            "ssm_suffix_topk": (ctypes.c_int, [vp, ctypes.c_int, i64, i64, i32, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -97,7 +98,7 @@ def exported_symbols() -> Sequence[str]:
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
             "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
-            "ssm_cache_append"]
+            "ssm_cache_append", "ssm_suffix_topk"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -254,6 +255,16 @@ def ssm_attention_varlen(q, k_new, v_new, pos, k_cache, v_cache, problems, n_pro
         _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(pos), _ptr(k_cache), _ptr(v_cache), total_new, total_cache,
         _ptr(problems), n_problems, max_n_new, max_n_cache, h_q, h_kv, d, float(rope_theta), float(scale),
         _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+# ------------------------------------------------------------------------------ suffix top-k
+
+
+def ssm_suffix_topk(logits, k: int, ids, probs, stream=None):
+    """logits: bf16/fp32 [n_rows, vocab]; ids int32 [n_rows, k]; probs fp32 [n_rows, k]."""
+    n_rows, vocab = logits.shape
+    _check("ssm_suffix_topk", lib().ssm_suffix_topk(
+        _ptr(logits), _dtype_code(logits), n_rows, vocab, int(k), _ptr(ids), _ptr(probs), _stream(stream)))
 
 
 # ------------------------------------------------------------------------------ prefix-cache append

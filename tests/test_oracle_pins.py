@@ -286,6 +286,47 @@ def test_rope_relative_position():
         assert abs(a - b) < 1e-10
 
 
+# ----------------------------------------------------------------------------- suffix top-k
+
+
+def test_suffix_topk_bruteforce_and_closed_forms():
+    # logits ln(1..6) on V = 6: probabilities are i / 21
+    l = np.log(np.array([[3.0, 1.0, 6.0, 2.0, 5.0, 4.0]]))
+    ids, probs = O.suffix_topk(l, 3)
+    assert ids.tolist() == [[2, 4, 5]]
+    assert np.allclose(probs, [[6 / 21, 5 / 21, 4 / 21]])
+    # all equal: the k lowest ids, each 1 / V
+    ids, probs = O.suffix_topk(np.zeros((2, 50)), 4)
+    assert ids.tolist() == [[0, 1, 2, 3]] * 2 and np.allclose(probs, 1 / 50)
+    # ties are broken by the lower id, and the order is by probability, not by id
+    ids, _ = O.suffix_topk(np.array([[0.0, 2.0, 1.0, 2.0, 1.0]]), 4)
+    assert ids.tolist() == [[1, 3, 2, 4]]
+    # one planted logit: p = 1 / (1 + (V - 1) e^-d)
+    V, d = 1000, 7.0
+    l = np.zeros((1, V))
+    l[0, 613] = d
+    ids, probs = O.suffix_topk(l, 2)
+    assert ids[0, 0] == 613 and np.isclose(probs[0, 0], 1 / (1 + (V - 1) * math.exp(-d)))
+    assert ids[0, 1] == 0 and np.isclose(probs[0, 1], math.exp(-d) * probs[0, 0])
+    with pytest.raises(ValueError):
+        O.suffix_topk(np.zeros((1, 3)), 4)
+
+
+def test_suffix_topk_agrees_with_unmask_confidence_and_sorting():
+    rng = np.random.default_rng(31)
+    l = np.round(rng.standard_normal((6, 300)) * 4, 2)
+    ids, probs = O.suffix_topk(l, 5)
+    for r in range(6):
+        conf, arg, p2 = O.token_confidence(l[r])
+        assert ids[r, 0] == arg and np.isclose(probs[r, 0], conf) and np.isclose(probs[r, 1], p2)
+        # against a full sort of the softmax (scipy-free: numpy argsort on (-p, id))
+        p = np.exp(l[r] - l[r].max())
+        p /= p.sum()
+        ref = np.lexsort((np.arange(300), -p))[:5]
+        assert ids[r].tolist() == ref.tolist() and np.allclose(probs[r], p[ref])
+    assert np.all(np.diff(probs, axis=1) <= 0) and np.all(probs.sum(1) <= 1 + 1e-12)
+
+
 # ----------------------------------------------------------------------------- prefix-cache append
 
 
