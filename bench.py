@@ -379,8 +379,14 @@ def _event_ms(fn, reps: int, warmup: int = 3) -> float:
     return e0.elapsed_time(e1) / reps
 
 
-def time_next_rows(w: W.Workload, n_suffix_rows: int, dev, hbm_peak: float) -> dict:
+def time_next_rows(inp: "StepInputs", attn_ms: float, dev, hbm_peak: float, tensor_peak: float) -> dict:
     """Secondary measurements of the rows that extend the step (not in the timed step).
+
+    unmask_margin / unmask_top1: the unmasking stage of the same step under the margin rule (which
+    needs the second-largest probability) and under Vanilla top-1 decoding.
+    full_suffix_attention: the attention the same block indices would need without structured
+    suffix modeling (every suffix position kept, the dense baseline), and the ratio to the step's
+    attention stage.
 
     suffix_topk: the next step's top-k candidates of every retained suffix position of one bench
     step (this workload's vocabulary, bf16 N(0, sigma) stand-in logits, read once).
@@ -388,8 +394,49 @@ def time_next_rows(w: W.Workload, n_suffix_rows: int, dev, hbm_peak: float) -> d
     K/V heads (one sequence; 268 MB moved, more than L2) appended into an 8192-row cache.
     """
     from paper_2608_23167_gb300 import ssm
+    w = inp.w
     out = {}
-    n = max(n_suffix_rows, 1)
+    p2 = torch.empty_like(inp.conf)
+    for name, kw in (("unmask_margin", dict(p2=p2, mode=ssm.SSM_COMMIT_MARGIN, threshold=w.threshold)),
+                     ("unmask_top1", dict(p2=None, mode=ssm.SSM_COMMIT_TOPK, topk=1))):
+        ms = _event_ms(lambda: ssm.ssm_unmask(inp.logits, inp.masked, inp.conf, inp.argmax, inp.commit,
+                                              workspace=inp.unmask_ws, **kw), reps=20)
+        out[name] = {"ms": ms, "GBps": inp.unmask_bytes() / (ms * 1e-3) / 1e9,
+                     "frac_hbm": inp.unmask_bytes() / (ms * 1e-3) / 1e9 / hbm_peak}
+    if inp.k_cache is not None and w.name == "long":
+        # every suffix position of every block index, against the same shared cache
+        rows, new_row = [], 0
+        for i, b in enumerate(w.block_indices):
+            n_new = w.block + (w.n_blocks - 1 - b) * w.block
+            rows.append((new_row, inp.cache_row[i], n_new, inp.n_cache[i]))
+            new_row += n_new
+        fq = W.draw_normal_bf16((new_row, w.h_q, w.head_dim), 1.0, 81, device=dev)
+        fk = W.draw_normal_bf16((new_row, w.h_kv, w.head_dim), 1.0, 82, device=dev)
+        fv = W.draw_normal_bf16((new_row, w.h_kv, w.head_dim), 1.0, 83, device=dev)
+        fpos = torch.cat([torch.arange(W.block_start(w, b), w.prompt + w.gen, dtype=torch.int32)
+                          for b in w.block_indices]).to(dev)
+        fo = torch.empty_like(fq)
+        ftab = ssm.attn_problems_tensor(rows, dev)
+        fws = torch.empty(ssm.ssm_attention_workspace_size(new_row, w.h_q, w.h_kv, w.head_dim), dtype=torch.uint8,
+                          device=dev)
+        max_rows = max(r[2] for r in rows)
+        ms = _event_ms(lambda: ssm.ssm_attention_varlen(fq, fk, fv, fpos, inp.k_cache, inp.v_cache, ftab, len(rows),
+                                                        max_rows, inp.max_cache, fo, w.rope_theta, workspace=fws),
+                       reps=5)
+        flops = 4.0 * w.h_q * w.head_dim * sum(r[2] * (r[2] + r[3]) for r in rows)
+        out["full_suffix_attention"] = {"rows": new_row, "ms": ms, "gflop": flops / 1e9,
+                                        "TFLOPs": flops / (ms * 1e-3) / 1e12,
+                                        "frac_bf16": flops / (ms * 1e-3) / 1e12 / tensor_peak,
+                                        "ssm_attention_ms": attn_ms, "attention_speedup": ms / attn_ms}
+        del fq, fk, fv, fo, fws
+    # early termination after a block: one sequence per block index of the sweep, the first block checked
+    toks = torch.randint(0, w.vocab - 1, (inp.n, w.gen), dtype=torch.int32, device=dev)
+    fin = torch.zeros(inp.n, dtype=torch.uint8, device=dev)
+    nact = torch.zeros(1, dtype=torch.int32, device=dev)
+    ms = _event_ms(lambda: ssm.ssm_early_stop(toks, w.block, 0, w.vocab - 2, fin, nact), reps=50)
+    out["early_stop"] = {"sequences": inp.n, "gen_len": w.gen, "us": ms * 1e3, "bound": "launch latency"}
+    del toks, fin, nact
+    n = max(inp.total_suffix, 1)
     lg = W.draw_logits((n, w.vocab), "bf16", w.logits_sigma, 73, device=dev)
     ids = torch.empty((n, w.topk), dtype=torch.int32, device=dev)
     pr = torch.empty((n, w.topk), dtype=torch.float32, device=dev)
@@ -559,7 +606,7 @@ def main():
 
     next_rows = None
     if rank == 0 and not args.no_next:
-        next_rows = time_next_rows(w, inp.total_suffix, dev, hbm_peak)
+        next_rows = time_next_rows(inp, attn_ms, dev, hbm_peak, tensor_peak)
         if ssm.ssm_get_device_error() != 0:
             raise RuntimeError("device error in the secondary measurements")
 

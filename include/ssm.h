@@ -12,8 +12,9 @@
  *   4. ssm_unmask             -- vocabulary softmax, confidence, argmax and the
  *                                threshold / top-k / margin commit (Sec. 4.2, 4.6)
  * and, around the step, ssm_suffix_topk (the retained suffix positions' top-k
- * candidates for the next step's Eq. 6) and ssm_cache_append (the prefix-cache
- * update at a block boundary, Sec. 4.8 "+PC.").
+ * candidates for the next step's Eq. 6), ssm_cache_append (the prefix-cache
+ * update at a block boundary, Sec. 4.8 "+PC.") and ssm_early_stop (early
+ * termination after a block, Sec. 3.2).
  *
  * Conventions (all entry points):
  *   - Every function returns ssm_status; nothing throws across the ABI.
@@ -330,6 +331,23 @@ ssm_status ssm_suffix_topk(const void* logits, ssm_dtype dtype, int64_t n_rows, 
 ssm_status ssm_cache_append(const void* k_new, const void* v_new, const int32_t* pos, int32_t batch,
                             int32_t n_rows, int32_t h_kv, int32_t head_dim, float rope_theta, void* k_cache,
                             void* v_cache, int64_t cache_rows, int64_t start_row, ssm_stream_t stream);
+
+/* ------------------------------------------------------------------------- */
+/* 6. Early termination after a decoded block (Sec. 3.2 "Early Termination"). */
+/* ------------------------------------------------------------------------- */
+
+/* For every sequence s with finished[s] == 0: if the generated tokens of block
+ * block_idx (positions block_idx*block_len .. +block_len-1 of tokens[s]) hold
+ * eos_id, set finished[s] = 1 and write eos_id at every generated position
+ * after the first EOS (the rest of that block and every later block).
+ * Sequences already finished are not touched.  n_active (optional, device
+ * int32) receives the number of sequences still running after the call.
+ *   tokens    int32 [batch, gen_len] (the generated region only), in place
+ *   finished  uint8 [batch], in place
+ * gen_len % block_len != 0 returns SSM_ERR_SHAPE; a block past the end returns
+ * SSM_ERR_INVALID_ARG. */
+ssm_status ssm_early_stop(int32_t* tokens, int32_t batch, int32_t gen_len, int32_t block_len, int32_t block_idx,
+                          int32_t eos_id, uint8_t* finished, int32_t* n_active, ssm_stream_t stream);
 
 #ifdef __cplusplus
 }

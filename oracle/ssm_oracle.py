@@ -24,6 +24,8 @@ in the paper's order:
                             softmax (Sec. 3.2 "Soft Suffix Embedding Mixing": the
                             set T^i_{t+1} and p^i_{t+1}(v) that Eq. 6 renormalizes
                             at the next step).
+* ``early_stop``         -- early termination after a decoded block (Sec. 3.2
+                            "Early Termination").
 * ``cache_append``       -- the prefix-cache update at a block boundary in the
                             prefix-caching setting ("+PC.", Sec. 4.8, Table 4):
                             the block's keys (rotated at their positions) and
@@ -289,6 +291,29 @@ def attention(q: np.ndarray, k_new: np.ndarray, v_new: np.ndarray, pos: np.ndarr
             out[bi, :, h, :] = (p @ vals[bi, :, g, :]) / l
             lse[bi, :, h] = (m + np.log(l))[:, 0]
     return out, lse
+
+
+def early_stop(tokens: np.ndarray, block_len: int, block_idx: int, eos_id: int, finished: np.ndarray):
+    """Early termination after block block_idx is decoded (Sec. 3.2 "Early Termination").
+
+    tokens: int [batch, gen_len], the generated region; finished: bool/uint8 [batch].
+    A running sequence whose block holds eos_id stops: it is marked finished and
+    every generated position after its first EOS becomes eos_id.  Readings: the
+    paper halts generation without saying what the positions after EOS hold; they
+    are filled with EOS, so no later block has a masked position left.  Returns
+    (tokens, finished, n_active) as new arrays.
+    """
+    tokens = np.array(tokens, copy=True)
+    finished = np.array(finished, dtype=np.uint8, copy=True)
+    b0, b1 = block_idx * block_len, (block_idx + 1) * block_len
+    for s in range(tokens.shape[0]):
+        if finished[s]:
+            continue
+        hits = [p for p in range(b0, b1) if tokens[s, p] == eos_id]
+        if hits:
+            finished[s] = 1
+            tokens[s, hits[0] + 1:] = eos_id
+    return tokens, finished, int(np.sum(finished == 0))
 
 
 def cache_append(k_cache: np.ndarray, v_cache: np.ndarray, k_new: np.ndarray, v_new: np.ndarray,

@@ -84,6 +84,7 @@ def lib() -> ctypes.CDLL:
                                                   i32, vp, vp, vp, vp, vp]),
             "ssm_cache_append": (ctypes.c_int, [vp, vp, vp, i32, i32, i32, i32, f32, vp, vp, i64, i64, vp]),
             "ssm_suffix_topk": (ctypes.c_int, [vp, ctypes.c_int, i64, i64, i32, vp, vp, vp]),
+            "ssm_early_stop": (ctypes.c_int, [vp, i32, i32, i32, i32, i32, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -98,7 +99,7 @@ def exported_symbols() -> Sequence[str]:
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
             "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
-            "ssm_cache_append", "ssm_suffix_topk"]
+            "ssm_cache_append", "ssm_suffix_topk", "ssm_early_stop"]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -265,6 +266,17 @@ def ssm_suffix_topk(logits, k: int, ids, probs, stream=None):
     n_rows, vocab = logits.shape
     _check("ssm_suffix_topk", lib().ssm_suffix_topk(
         _ptr(logits), _dtype_code(logits), n_rows, vocab, int(k), _ptr(ids), _ptr(probs), _stream(stream)))
+
+
+# ------------------------------------------------------------------------------ early termination
+
+
+def ssm_early_stop(tokens, block_len: int, block_idx: int, eos_id: int, finished, n_active=None, stream=None):
+    """tokens: int32 [batch, gen_len] (in place); finished: uint8 [batch] (in place); n_active: int32 [1]."""
+    batch, gen_len = tokens.shape
+    _check("ssm_early_stop", lib().ssm_early_stop(
+        _ptr(tokens), batch, gen_len, int(block_len), int(block_idx), int(eos_id), _ptr(finished), _ptr(n_active),
+        _stream(stream)))
 
 
 # ------------------------------------------------------------------------------ prefix-cache append

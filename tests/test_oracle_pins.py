@@ -327,6 +327,31 @@ def test_suffix_topk_agrees_with_unmask_confidence_and_sorting():
     assert np.all(np.diff(probs, axis=1) <= 0) and np.all(probs.sum(1) <= 1 + 1e-12)
 
 
+# ----------------------------------------------------------------------------- early termination
+
+
+def test_early_stop_hand_cases():
+    E = 9
+    toks = np.array([[1, 2, 3, 4, 5, 6, 7, 8],     # no EOS in block 1 (positions 4..7): still running
+                     [1, 2, 3, 4, 5, E, 7, 8],     # EOS at 5: 6, 7 become EOS
+                     [1, E, 3, 4, 5, 6, 7, 8],     # EOS only in block 0, not the checked block: running
+                     [1, 2, 3, 4, E, 6, E, 8],     # first EOS of the block at 4 decides
+                     [1, 2, 3, 4, 5, 6, 7, E]])    # EOS at the block's last position: nothing to fill
+    fin = np.array([0, 0, 0, 0, 0], dtype=np.uint8)
+    t, f, n = O.early_stop(toks, 4, 1, E, fin)
+    assert f.tolist() == [0, 1, 0, 1, 1] and n == 2
+    assert t[0].tolist() == toks[0].tolist() and t[2].tolist() == toks[2].tolist()
+    assert t[1].tolist() == [1, 2, 3, 4, 5, E, E, E]
+    assert t[3].tolist() == [1, 2, 3, 4, E, E, E, E]
+    assert t[4].tolist() == toks[4].tolist()
+    # a finished sequence is not touched, even with an EOS in the block
+    t2, f2, n2 = O.early_stop(toks, 4, 1, E, np.array([1, 1, 1, 1, 1], dtype=np.uint8))
+    assert np.array_equal(t2, toks) and f2.tolist() == [1] * 5 and n2 == 0
+    # filling reaches later blocks: block 0 of 3
+    t3, f3, _ = O.early_stop(np.array([[E, 5, 5, 5, 5, 5]]), 2, 0, E, np.array([0], dtype=np.uint8))
+    assert t3.tolist() == [[E] * 6] and f3.tolist() == [1]
+
+
 # ----------------------------------------------------------------------------- prefix-cache append
 
 
