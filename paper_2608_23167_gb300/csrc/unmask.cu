@@ -126,8 +126,9 @@ struct RunState {
   int idx;
 };
 
+// (with the second largest tracked, the register cap keeps four CTAs per SM)
 template <typename T, bool NEED_SECOND>
-__global__ void __launch_bounds__(kStreamThreads) unmask_stream_kernel(
+__global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_stream_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part, unsigned* err, uint64_t wait_ns) {
   constexpr int ESZ = sizeof(T);
@@ -207,14 +208,20 @@ __global__ void __launch_bounds__(kStreamThreads) unmask_stream_kernel(
       }
       const float cm1 = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
       if constexpr (NEED_SECOND) {
-        float s2 = -INFINITY, m1l = -INFINITY;
+        // second largest of the running values after this chunk (a repeated maximum counts
+        // twice): only a chunk that raises the maximum needs its own second largest, which
+        // is rare once the row is under way
+        if (cm1 > r.m1) {
+          float s2 = -INFINITY, m1l = -INFINITY;
 #pragma unroll
-        for (int e = 0; e < PER; ++e) {
-          s2 = fmaxf(s2, fminf(m1l, f[e]));
-          m1l = fmaxf(m1l, f[e]);
+          for (int e = 0; e < PER; ++e) {
+            s2 = fmaxf(s2, fminf(m1l, f[e]));
+            m1l = fmaxf(m1l, f[e]);
+          }
+          r.m2 = fmaxf(fmaxf(r.m1, s2), r.m2);
+        } else {
+          r.m2 = fmaxf(r.m2, cm1);
         }
-        // second largest of the running values after this chunk (a repeated maximum counts twice)
-        r.m2 = (cm1 > r.m1) ? fmaxf(fmaxf(r.m1, s2), r.m2) : fmaxf(r.m2, cm1);
       }
       if (cm1 > r.m1) {
         if (r.m1 > -INFINITY) r.s *= ex2((r.m1 - cm1) * kLog2e);
