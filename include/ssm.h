@@ -306,7 +306,9 @@ ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, int32_t batch
  *              element size a multiple of 16 and logits 16-byte aligned;
  *              otherwise SSM_ERR_UNSUPPORTED)
  *   ids        int32 [n_rows, k];  probs  fp32 [n_rows, k]
- * 1 <= k <= 8 (SSM_ERR_UNSUPPORTED otherwise), k <= vocab.  No workspace. */
+ * 1 <= k <= 8 (SSM_ERR_UNSUPPORTED otherwise), k <= vocab; vocab up to
+ * 2,744,320 (bf16) or 684,032 (fp32) entries (a row's per-slice maxima are kept
+ * in shared memory; SSM_ERR_UNSUPPORTED beyond).  No workspace. */
 ssm_status ssm_suffix_topk(const void* logits, ssm_dtype dtype, int64_t n_rows, int64_t vocab, int32_t k,
                            int32_t* ids, float* probs, ssm_stream_t stream);
 

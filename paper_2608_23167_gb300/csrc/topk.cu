@@ -5,12 +5,13 @@
 // ids (ties: lower id first) and their full-vocabulary softmax probabilities.
 //
 // topk_row_kernel: the unmasking pass's streaming scheme (stream.cuh), one
-// row per CTA at a time, with a threshold that keeps the candidate lists idle
-// after the row's first chunk (see the kernel).
+// row per CTA at a time, read once; the few slices that can hold a candidate
+// are re-read at the row's end (see the kernel).
 #include <cuda_bf16.h>
 
 #include <algorithm>
 #include <atomic>
+#include <type_traits>
 
 #include "common.cuh"
 #include "sm100_ptx.cuh"
@@ -25,6 +26,7 @@ constexpr int kTopStageBytes = 16384;      // one chunk: 64 bytes per thread
 constexpr int kTopStages = 2;
 constexpr int kTopVecPerThread = kTopStageBytes / 16 / kTopThreads;  // 4
 constexpr float kLog2eT = 1.4426950408889634f;
+constexpr int64_t kTopMaxSmem = 200 * 1024;   // dynamic shared memory cap: bf16 rows up to 2,744,320 entries, fp32 684,032
 
 __device__ __forceinline__ float ex2t(float x) {
   float y;
@@ -50,14 +52,6 @@ __device__ __forceinline__ void list_insert(float (&v)[kTopMax], int (&id)[kTopM
     v[0] = x;
     id[0] = ix;
   }
-}
-
-__device__ __forceinline__ void ms_merge(float& m, float& s, float m2, float s2) {
-  const float mm = fmaxf(m, m2);
-  const float a = (s > 0.f) ? s * ex2t((m - mm) * kLog2eT) : 0.f;
-  const float b = (s2 > 0.f) ? s2 * ex2t((m2 - mm) * kLog2eT) : 0.f;
-  m = mm;
-  s = a + b;
 }
 
 // Each warp's k best (value, id) among its lanes' decreasing lists of L entries
@@ -104,8 +98,9 @@ __device__ __forceinline__ void warp_topk(const float (&lv)[L], const int (&li)[
 }
 
 // The k best of the eight warps' lists in wv / wi (k rounds over their heads);
-// returns the k-th value and, if out_v is given, writes the k (value, id).
-__device__ __forceinline__ float merge_warp_lists(const float* wv, const int* wi, int k, float* out_v,
+// returns the k-th value, sets top to the best one and, if out_v is given,
+// writes the k (value, id).
+__device__ __forceinline__ float merge_warp_lists(const float* wv, const int* wi, int k, float& top, float* out_v,
                                                   int* out_i) {
   int head[kTopThreads / 32];
 #pragma unroll
@@ -133,136 +128,165 @@ __device__ __forceinline__ float merge_warp_lists(const float* wv, const int* wi
       out_v[r] = bv;
       out_i[r] = bi;
     }
+    if (r == 0) top = bv;
     t = bv;
   }
   return t;
 }
 
-// The row's k-th best value so far among all lanes' lists, as a lower bound:
-// every thread of the CTA gets it (one barrier pair).
-template <int L>
-__device__ __forceinline__ float block_kth(const float (&lv)[L], const int (&li)[L], int k, float* wv, int* wi) {
-  warp_topk<L>(lv, li, k, wv, wi);
-  __syncthreads();
-  const float t = merge_warp_lists(wv, wi, k, nullptr, nullptr);
-  __syncthreads();
-  return t;
+__device__ __forceinline__ void ms_merge(float& m, float& s, float m2, float s2) {
+  const float mm = fmaxf(m, m2);
+  const float a = (s > 0.f) ? s * ex2t((m - mm) * kLog2eT) : 0.f;
+  const float b = (s2 > 0.f) ? s2 * ex2t((m2 - mm) * kLog2eT) : 0.f;
+  m = mm;
+  s = a + b;
 }
 
-// One CTA per row at a time (rows dealt round-robin to persistent CTAs).  The
-// row streams through the cp.async ring; every thread keeps (max, sum of exp)
-// and a decreasing list of its 8 best (value, id).  A threshold T bounds the
-// row's k-th best value from below: first the k-th largest of the threads'
-// maxima of chunk 0, then, after chunks 1 and 3, the k-th best entry of all
-// lists (k distinct entries of the row reach it either way).  Nothing below T
-// can be a candidate, and a chunk touches a list only for a value >= T that
-// ranks before the list's last entry, which soon becomes rare.  At the
-// row's end each warp takes its k best by k rounds of warp argmax and one
-// thread merges the eight lists.
+// Order-preserving map of a float to an unsigned key (larger float, larger key).
+__device__ __forceinline__ uint32_t float_key(float x) {
+  const uint32_t b = __float_as_uint(x);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(uint32_t key) {
+  return __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key);
+}
+
+// The k-th largest (with multiplicity) and the largest of the CTA's 256 values
+// x, for every thread (one barrier; red holds 8 x kTopMax keys and must not be
+// rewritten before the CTA's next barrier).  Each warp writes its k largest
+// keys by rounds of warp max, each round taking the lanes that hold the
+// maximum; then every warp takes the k-th largest of the written keys the same way.
+__device__ __forceinline__ float block_kth(float x, int k, float& top, uint32_t* red) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint32_t key = float_key(x);
+  for (int above = 0; above < k;) {
+    const uint32_t mx = __reduce_max_sync(0xffffffffu, key);
+    const uint32_t ball = __ballot_sync(0xffffffffu, key == mx);
+    if (key == mx) {
+      const int slot = above + __popc(ball & ((1u << lane) - 1u));
+      if (slot < k) red[warp * kTopMax + slot] = mx;
+      key = 0u;
+    }
+    above += __popc(ball);
+  }
+  __syncthreads();
+  // lane l holds slots 2l and 2l + 1 of the 8 x kTopMax table (slots >= k unused: key 0)
+  uint32_t a = ((2 * lane) % kTopMax < k) ? red[2 * lane] : 0u;
+  uint32_t b = ((2 * lane + 1) % kTopMax < k) ? red[2 * lane + 1] : 0u;
+  uint32_t res = 0u;
+  for (int above = 0, r = 0; above < k; ++r) {
+    const uint32_t mx = __reduce_max_sync(0xffffffffu, max(a, b));
+    if (r == 0) top = key_float(mx);
+    above += __popc(__ballot_sync(0xffffffffu, a == mx)) + __popc(__ballot_sync(0xffffffffu, b == mx));
+    res = mx;
+    if (a == mx) a = 0u;
+    if (b == mx) b = 0u;
+  }
+  return key_float(res);
+}
+
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
+// A thread's 64 bytes of one chunk are 16 words w[4u + q] (its vector u, word q);
+// entry h of word (u, q) is  chunk_start + (u * threads + thread) * epv + q * (epv / 4) + h.
+template <typename T>
+__device__ __forceinline__ float words_max(const uint32_t (&w)[16]) {
+  if constexpr (sizeof(T) == 2) {
+    uint32_t x[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) x[c] = bmax2(bmax2(w[c], w[4 + c]), bmax2(w[8 + c], w[12 + c]));
+    const uint32_t y = bmax2(bmax2(x[0], x[1]), bmax2(x[2], x[3]));
+    return fmaxf(lo_bf16(y), hi_bf16(y));
+  } else {
+    float a = fmax3(__uint_as_float(w[0]), __uint_as_float(w[1]), __uint_as_float(w[2]));
+    float b = fmax3(__uint_as_float(w[3]), __uint_as_float(w[4]), __uint_as_float(w[5]));
+    a = fmax3(a, __uint_as_float(w[6]), __uint_as_float(w[7]));
+    b = fmax3(b, __uint_as_float(w[8]), __uint_as_float(w[9]));
+    a = fmax3(a, __uint_as_float(w[10]), __uint_as_float(w[11]));
+    b = fmax3(b, __uint_as_float(w[12]), __uint_as_float(w[13]));
+    return fmax3(a, b, fmaxf(__uint_as_float(w[14]), __uint_as_float(w[15])));
+  }
+}
+
+// One CTA per row at a time (rows dealt round-robin to persistent CTAs), the row
+// streamed once through the unmasking pass's cp.async ring (stream.cuh).  Each
+// thread folds its 64 bytes of a chunk into a running (max m, sum of exp(x - m))
+// and records the slice's maximum in shared memory.  At the row's end the CTA
+// fixes T = the k-th largest of the threads' maxima: k distinct entries reach T,
+// so the row's k-th best value is >= T and only slices whose maximum reaches T
+// can hold a candidate (on random logits about k of the row's 4096 slices).  Each
+// thread re-reads those of its slices from global memory and keeps a decreasing
+// list of its 8 best (value, id) among their entries >= T; each warp then takes
+// its k best by k rounds of warp argmax and one thread merges the eight lists.
 template <typename T>
 __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restrict__ logits, int64_t vocab,
                                                               int64_t n_rows, int k, int32_t* __restrict__ ids,
                                                               float* __restrict__ probs) {
   constexpr int ESZ = sizeof(T);
-  constexpr int EPV = 16 / ESZ;                       // elements per 16-byte vector
-  constexpr int PER = kTopVecPerThread * EPV;         // values per thread and chunk
+  constexpr int EPV = 16 / ESZ;          // entries per 16-byte vector
+  constexpr int EPW = EPV / 4;           // entries per word
+  constexpr int EPC = kTopStageBytes / ESZ;   // entries per chunk
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+  // [chunk][thread] slice maxima, stored in the logits' own type (exact)
+  using Slice = typename std::conditional<ESZ == 2, uint16_t, uint32_t>::type;
+  Slice* slice_max = reinterpret_cast<Slice*>(ring + kTopStages * kTopStageBytes);
   __shared__ float red_m[kTopThreads / 32], red_s[kTopThreads / 32];
   __shared__ float red_kv[(kTopThreads / 32) * kTopMax];
   __shared__ int red_ki[(kTopThreads / 32) * kTopMax];
+  __shared__ uint32_t red_key[(kTopThreads / 32) * kTopMax];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  ChunkIter is{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
-  chunk_seek<T>(is, vocab, vocab, 1, n_rows, nullptr);
+  const int64_t row_bytes = vocab * ESZ;
+  const int nchunk = static_cast<int>((row_bytes + kTopStageBytes - 1) / kTopStageBytes);
+  const uint32_t ninf = (ESZ == 2) ? 0xFF80FF80u : 0xFF800000u;
+  int64_t irow = blockIdx.x;
+  int ichunk = 0;
   auto issue = [&](int slot) {
-    if (is.valid) {
-      const uint8_t* src = reinterpret_cast<const uint8_t*>(logits + is.row * vocab) + is.off;
+    if (irow < n_rows) {
+      const int64_t off = static_cast<int64_t>(ichunk) * kTopStageBytes;
+      const uint8_t* src = reinterpret_cast<const uint8_t*>(logits + irow * vocab) + off;
       uint8_t* dst = ring + slot * kTopStageBytes;
 #pragma unroll
       for (int u = 0; u < kTopVecPerThread; ++u) {
         const int vi = u * kTopThreads + threadIdx.x;
-        if (vi * 16 < is.bytes - is.off) cp_async16(dst + vi * 16, src + vi * 16);
+        if (vi * 16 < row_bytes - off) cp_async16(dst + vi * 16, src + vi * 16);
       }
-      is.off += kTopStageBytes;
-      chunk_seek<T>(is, vocab, vocab, 1, n_rows, nullptr);
+      if (++ichunk == nchunk) {
+        ichunk = 0;
+        irow += gridDim.x;
+      }
     }
     cp_async_commit();
   };
 #pragma unroll
   for (int q = 0; q < kTopStages; ++q) issue(q);
 
-  ChunkIter cs{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
-  chunk_seek<T>(cs, vocab, vocab, 1, n_rows, nullptr);
   int slot = 0;
-  while (cs.valid) {
-    const int64_t row = cs.item;
-    float m = -INFINITY, s = 0.f, thr = -INFINITY;
-    float tv[kTopMax];
-    int ti[kTopMax];
-#pragma unroll
-    for (int j = 0; j < kTopMax; ++j) {
-      tv[j] = -INFINITY;
-      ti[j] = INT_MAX;
-    }
-    int nchunk = 0;  // chunks of this row done
-    while (cs.valid && cs.item == row) {
+  for (int64_t row = blockIdx.x; row < n_rows; row += gridDim.x) {
+    float m = -INFINITY, s = 0.f;
+    for (int c = 0; c < nchunk; ++c) {
       cp_async_wait<kTopStages - 1>();
-      const int chunk_bytes = static_cast<int>(min(static_cast<int64_t>(kTopStageBytes), cs.bytes - cs.off));
+      const int64_t off = static_cast<int64_t>(c) * kTopStageBytes;
+      const int chunk_bytes = static_cast<int>(min(static_cast<int64_t>(kTopStageBytes), row_bytes - off));
       const uint4* sv = reinterpret_cast<const uint4*>(ring + slot * kTopStageBytes);
-      const uint32_t ninf = (ESZ == 2) ? 0xFF80FF80u : 0xFF800000u;
-      float f[PER];
+      uint32_t w[16];
 #pragma unroll
       for (int u = 0; u < kTopVecPerThread; ++u) {
         const int vi = u * kTopThreads + threadIdx.x;
         const uint4 v = vi * 16 < chunk_bytes ? sv[vi] : make_uint4(ninf, ninf, ninf, ninf);
-        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          if constexpr (ESZ == 2) {
-            f[u * 8 + 2 * q] = lo_bf16(w4[q]);
-            f[u * 8 + 2 * q + 1] = hi_bf16(w4[q]);
-          } else {
-            f[u * 4 + q] = __uint_as_float(w4[q]);
-          }
-        }
+        w[4 * u] = v.x;
+        w[4 * u + 1] = v.y;
+        w[4 * u + 2] = v.z;
+        w[4 * u + 3] = v.w;
       }
-      float c4[4] = {f[0], f[1], f[2], f[3]};
-#pragma unroll
-      for (int e = 4; e < PER; e += 8) {
-        c4[0] = fmax3(c4[0], f[e], f[e + 1]);
-        c4[1] = fmax3(c4[1], f[e + 2], f[e + 3]);
-        if (e + 4 < PER) {
-          c4[2] = fmax3(c4[2], f[e + 4], f[e + 5]);
-          c4[3] = fmax3(c4[3], f[e + 6], f[e + 7]);
-        }
-      }
-      const float cm = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
-      if (nchunk == 0) {
-        // before any list work: T = the k-th largest of the threads' chunk maxima
-        const float one[1] = {cm};
-        const int tag[1] = {static_cast<int>(threadIdx.x)};   // distinct per thread: only the value is used
-        thr = block_kth<1>(one, tag, k, red_kv, red_ki);
-      }
-      // a value enters the list only when it reaches the threshold and ranks before the
-      // list's last entry
-      if (cm >= thr && cm >= tv[kTopMax - 1]) {
-        const int tbase = static_cast<int>(cs.off / ESZ) + static_cast<int>(threadIdx.x) * EPV;
-        // scan only the max chains whose maximum qualifies (chain q holds e = q and the pairs
-        // 4 + 8i + 2q, 5 + 8i + 2q of the reduction above); chains are visited out of id
-        // order, so an entry is compared with the list's last one by (value, id)
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          if (c4[q] >= thr && c4[q] >= tv[kTopMax - 1]) {
-#pragma unroll
-            for (int e = 0; e < PER; ++e) {
-              const bool in_chain = (e < 4) ? (e == q) : (((e - 4) % 8) / 2 == q);
-              const int id = tbase + (e / EPV) * kTopThreads * EPV + (e % EPV);
-              if (in_chain && f[e] >= thr && better(f[e], id, tv[kTopMax - 1], ti[kTopMax - 1]))
-                list_insert(tv, ti, f[e], id);
-            }
-          }
-        }
-      }
+      issue(slot);
+      slot = (slot + 1) % kTopStages;
+      const float cm = words_max<T>(w);
+      slice_max[c * kTopThreads + threadIdx.x] = static_cast<Slice>(__float_as_uint(cm) >> (32 - 8 * ESZ));
       if (cm > m) {
         if (m > -INFINITY) s *= ex2t((m - cm) * kLog2eT);
         m = cm;
@@ -271,37 +295,71 @@ __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restri
         const float mb = m * kLog2eT;
         float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int e = 0; e < PER; e += 2) {
+        for (int e = 0; e < 16; e += (ESZ == 2 ? 1 : 2)) {
+          float x0, x1;
+          if constexpr (ESZ == 2) {
+            x0 = lo_bf16(w[e]);
+            x1 = hi_bf16(w[e]);
+          } else {
+            x0 = __uint_as_float(w[e]);
+            x1 = __uint_as_float(w[e + 1]);
+          }
           float t0, t1;
-          ffma2(t0, t1, f[e], f[e + 1], kLog2eT, kLog2eT, -mb, -mb);
-          fadd2_acc(sa[(e >> 1) & 3], sb[(e >> 1) & 3], ex2t(t0), ex2t(t1));
+          ffma2(t0, t1, x0, x1, kLog2eT, kLog2eT, -mb, -mb);
+          const int a = (ESZ == 2 ? e : e >> 1) & 3;
+          fadd2_acc(sa[a], sb[a], ex2t(t0), ex2t(t1));
         }
         s += ((sa[0] + sb[0]) + (sa[1] + sb[1])) + ((sa[2] + sb[2]) + (sa[3] + sb[3]));
       }
-      issue(slot);
-      slot = (slot + 1) % kTopStages;
-      cs.off += kTopStageBytes;
-      if (cs.off >= cs.bytes) chunk_seek<T>(cs, vocab, vocab, 1, n_rows, nullptr);
-      if (nchunk == 1 || nchunk == 3) thr = fmaxf(thr, block_kth<kTopMax>(tv, ti, k, red_kv, red_ki));
-      ++nchunk;
     }
-    // the row's (max, sum)
+    // T, then the candidates of the slices whose maximum reaches it
+    float top;
+    const float thr = block_kth(m, k, top, red_key);
+    float tv[kTopMax];
+    int ti[kTopMax];
+#pragma unroll
+    for (int j = 0; j < kTopMax; ++j) {
+      tv[j] = -INFINITY;
+      ti[j] = INT_MAX;
+    }
+    for (int c = 0; c < nchunk; ++c) {
+      if (__uint_as_float(static_cast<uint32_t>(slice_max[c * kTopThreads + threadIdx.x]) << (32 - 8 * ESZ)) < thr)
+        continue;
+      const int64_t off = static_cast<int64_t>(c) * kTopStageBytes;
+      const int chunk_bytes = static_cast<int>(min(static_cast<int64_t>(kTopStageBytes), row_bytes - off));
+      const uint4* gv = reinterpret_cast<const uint4*>(reinterpret_cast<const uint8_t*>(logits + row * vocab) + off);
+#pragma unroll
+      for (int u = 0; u < kTopVecPerThread; ++u) {
+        const int vi = u * kTopThreads + threadIdx.x;
+        const uint4 v = vi * 16 < chunk_bytes ? __ldg(gv + vi) : make_uint4(ninf, ninf, ninf, ninf);
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+          for (int h = 0; h < EPW; ++h) {
+            const float f = (ESZ == 2) ? (h ? hi_bf16(w4[q]) : lo_bf16(w4[q])) : __uint_as_float(w4[q]);
+            const int id = c * EPC + vi * EPV + q * EPW + h;
+            if (f >= thr && better(f, id, tv[kTopMax - 1], ti[kTopMax - 1])) list_insert(tv, ti, f, id);
+          }
+        }
+      }
+    }
+    // the row's (max, sum) and its k best
 #pragma unroll
     for (int d = 16; d >= 1; d >>= 1) ms_merge(m, s, __shfl_xor_sync(0xffffffffu, m, d), __shfl_xor_sync(0xffffffffu, s, d));
     if (lane == 0) {
       red_m[warp] = m;
       red_s[warp] = s;
     }
-    // the row's k best: the warps' k best, then thread 0 merges them
     warp_topk<kTopMax>(tv, ti, k, red_kv, red_ki);
     __syncthreads();
     if (threadIdx.x == 0) {
       float rm = red_m[0], rs = red_s[0];
-      for (int w = 1; w < kTopThreads / 32; ++w) ms_merge(rm, rs, red_m[w], red_s[w]);
+      for (int q = 1; q < kTopThreads / 32; ++q) ms_merge(rm, rs, red_m[q], red_s[q]);
       const float inv = 1.f / rs;
-      float bv[kTopMax];
+      float bv[kTopMax], best;
       int bi[kTopMax];
-      merge_warp_lists(red_kv, red_ki, k, bv, bi);
+      merge_warp_lists(red_kv, red_ki, k, best, bv, bi);
       for (int r = 0; r < k; ++r) {
         ids[row * k + r] = bi[r];
         probs[row * k + r] = ex2t((bv[r] - rm) * kLog2eT) * inv;
@@ -344,8 +402,12 @@ ssm_status ssm_suffix_topk(const void* logits, ssm_dtype dtype, int64_t n_rows, 
   // 16-byte copies need 16-byte aligned rows
   if (!ssm::aligned16(logits) || (vocab * esz) % 16 != 0) return SSM_ERR_UNSUPPORTED;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const size_t smem = ssm::kTopStages * ssm::kTopStageBytes + 128;
-  const int grid = static_cast<int>(std::min<int64_t>(n_rows, 6ll * ssm::num_sms()));
+  // the ring plus one logit per (chunk, thread): the row's slice maxima
+  const int64_t nchunk = (vocab * esz + ssm::kTopStageBytes - 1) / ssm::kTopStageBytes;
+  const int64_t smem64 = ssm::kTopStages * ssm::kTopStageBytes + nchunk * ssm::kTopThreads * esz + 128;
+  if (smem64 > ssm::kTopMaxSmem) return SSM_ERR_UNSUPPORTED;
+  const size_t smem = static_cast<size_t>(smem64);
+  const int grid = static_cast<int>(std::min<int64_t>(n_rows, 5ll * ssm::num_sms()));
   if (dtype == SSM_DTYPE_BF16) {
     if (!ssm::topk_attr_set<ssm::topk_row_kernel<__nv_bfloat16>>(smem)) return SSM_ERR_CUDA;
     ssm::topk_row_kernel<__nv_bfloat16><<<grid, ssm::kTopThreads, smem, st>>>(

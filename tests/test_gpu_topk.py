@@ -92,5 +92,8 @@ def test_topk_errors(dev):
     with pytest.raises(ssm.SSMError) as e:
         ssm.ssm_suffix_topk(torch.zeros((2, 4099), dtype=torch.bfloat16, device=dev), 5, ids, pr)
     assert e.value.status == ssm.SSM_ERR_UNSUPPORTED          # rows not 16-byte multiples
+    with pytest.raises(ssm.SSMError) as e:
+        ssm.ssm_suffix_topk(torch.zeros((2, 3 << 20), dtype=torch.bfloat16, device=dev), 5, ids, pr)
+    assert e.value.status == ssm.SSM_ERR_UNSUPPORTED          # a row's slice maxima exceed shared memory
     ssm.ssm_suffix_topk(x[:0], 5, ids, pr)                      # no rows: nothing to do
     check_device_error()
