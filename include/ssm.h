@@ -276,9 +276,9 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
  * scratch is a fixed 1 MiB array in device global memory that the library
  * holds on every GPU that loads it, until the process exits.
  *   - Limit: ssm_unmask_workspace_size(batch, block_len, vocab, dtype) must be
- *     at most 1 MiB (for example batch * block_len <= 16384 positions with a
- *     126464-entry bf16 vocabulary); larger calls return SSM_ERR_CAPACITY and
- *     enqueue nothing.
+ *     at most 1 MiB (with a 126464-entry bf16 vocabulary that holds every
+ *     call of up to 65535 positions, the most ssm_unmask takes); larger calls
+ *     return SSM_ERR_CAPACITY and enqueue nothing.
  *   - The first call on a device looks up the array's device address (with
  *     that device current); make that first call before any stream capture.
  *   - Every call shares the one array: two calls that overlap on the GPU (on

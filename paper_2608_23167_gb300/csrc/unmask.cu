@@ -2,8 +2,9 @@
 // and parallel threshold decoding; Sec. 4.6: margin decoding).
 //
 // Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
-// segments of 32768 entries (the work items, dealt round-robin to persistent
-// CTAs, six per SM).  Each thread streams its own 64-byte slices of successive
+// segments of whole 16 KB chunks (the work items, dealt round-robin to
+// persistent CTAs, six per SM): one segment per row once a call has 2048 rows,
+// shorter ones for smaller calls.  Each thread streams its own 64-byte slices of successive
 // 16 KB chunks from HBM into a private two-stage shared-memory ring with
 // 16-byte cp.async copies, so the read runs ahead of the arithmetic without any
 // barrier (a thread only reads back what it copied itself), and folds every
@@ -29,7 +30,7 @@ namespace ssm {
 namespace {
 
 constexpr int kUnmaskThreads = 256;
-constexpr int kUnroll = 16;                        // a segment is 256 x 16 vectors of 16 bytes
+constexpr int64_t kItemsTarget = 2048;             // segments (work items) a call aims for
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Partial {
@@ -375,13 +376,21 @@ struct UnmaskPlan {
   bool vector;
 };
 
-UnmaskPlan plan_unmask(int64_t vocab, ssm_dtype dtype, const void* logits) {
+// Segments are whole 16 KB stages.  A row is cut into the fewest segments that
+// still give about kItemsTarget work items over all rows: one segment per row
+// once there are that many rows (every segment ends in a CTA-wide merge, so
+// fewer, longer segments stream faster), more for small calls so that their
+// rows still spread over the SMs.
+UnmaskPlan plan_unmask(int64_t rows, int64_t vocab, ssm_dtype dtype, const void* logits) {
   const int esz = dtype == SSM_DTYPE_BF16 ? 2 : 4;
-  const int vec = 16 / esz;
   UnmaskPlan p;
   p.vector = ((vocab * esz) % 16 == 0) && (logits == nullptr || ssm::aligned16(logits));
-  // both plans cut a row into the same chunks, so the workspace does not depend on the plan
-  p.chunk = static_cast<int64_t>(ssm::kUnmaskThreads) * ssm::kUnroll * vec;  // 64 KB segments
+  // both plans cut a row into the same segments, so the workspace does not depend on the plan
+  const int64_t stage_elems = ssm::kStageBytes / esz;
+  const int64_t n_stage = (vocab + stage_elems - 1) / stage_elems;
+  const int64_t per_row = (ssm::kItemsTarget + rows - 1) / std::max<int64_t>(rows, 1);
+  const int64_t want = std::min<int64_t>(std::max<int64_t>(per_row, 1), n_stage);
+  p.chunk = ((n_stage + want - 1) / want) * stage_elems;
   p.n_chunks = static_cast<int>((vocab + p.chunk - 1) / p.chunk);
   return p;
 }
@@ -408,7 +417,7 @@ extern "C" {
 
 size_t ssm_unmask_workspace_size(int32_t batch, int32_t block_len, int64_t vocab, ssm_dtype dtype) {
   if (batch <= 0 || block_len <= 0 || vocab <= 0) return 0;
-  const UnmaskPlan plan = plan_unmask(vocab, dtype, nullptr);
+  const UnmaskPlan plan = plan_unmask(static_cast<int64_t>(batch) * block_len, vocab, dtype, nullptr);
   return ssm::align_up(static_cast<size_t>(batch) * block_len * plan.n_chunks * sizeof(ssm::Partial), 256);
 }
 
@@ -430,7 +439,7 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   if (ws_bytes < ssm_unmask_workspace_size(batch, block_len, vocab, dtype)) return SSM_ERR_CAPACITY;
   const int64_t rows = static_cast<int64_t>(batch) * block_len;
   if (rows > 65535) return SSM_ERR_UNSUPPORTED;
-  const UnmaskPlan plan = plan_unmask(vocab, dtype, logits);
+  const UnmaskPlan plan = plan_unmask(rows, vocab, dtype, logits);
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));

@@ -91,5 +91,8 @@ def test_workspace_sizes(lib):
     from paper_2608_23167_gb300 import ssm
     import torch
     assert ssm.ssm_attention_workspace_size(101 * 8, 32, 32, 128) == 2 * 101 * 8 * 32 * 128 * 2
+    # 126464 bf16 entries are 16 stages of 8192; segments aim at 2048 work items per call
     ws = ssm.ssm_unmask_workspace_size(8, 32, 126464, torch.bfloat16)
-    assert ws == 8 * 32 * 4 * 16   # four 32768-entry chunks per row, 16-byte partials
+    assert ws == 8 * 32 * 8 * 16   # 256 rows: eight segments of two stages each, 16-byte partials
+    assert ssm.ssm_unmask_workspace_size(64, 32, 126464, torch.bfloat16) == 64 * 32 * 16   # one segment per row
+    assert ssm.ssm_unmask_workspace_size(1, 4, 126464, torch.bfloat16) == 4 * 16 * 16      # one stage per segment
