@@ -138,62 +138,78 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 constexpr int kRopeWarps = 8;
 
-// One warp per new row.  Each lane owns four rotation pairs (i, i + D/2) of one
-// head vector, so D/8 lanes cover a head and a warp moves 32/(D/8) heads per
-// pass with 8-byte loads and stores.  The rotation is rope.cuh's (inverse
-// frequencies once per CTA).
+// Persistent warps over (problem, row) items, item = problem * rows_per_problem_max
+// + row (items past a problem's row count are skipped).  A row's D/2 angles are
+// formed once (two per lane) and shared through shared memory; a lane then owns
+// eight rotation pairs (i, i + D/2) of one head vector (D/16 lanes per head,
+// 16-byte loads and stores, two head passes in flight).  The rotation is
+// rope.cuh's (inverse frequencies once per CTA).
 template <int D>
 __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
-    const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max,
+    const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max, int32_t n_prob,
     __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
-  constexpr int LPH = D / 8;        // lanes per head vector
+  constexpr int LPH = D / 16;       // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
+  __shared__ float s_cs[kRopeWarps][D / 2], s_sn[kRopeWarps][D / 2];
   if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int sub = lane % LPH;       // which 4 pairs
-  const int hoff = lane / LPH;      // which head of the pass
-  const int prob = blockIdx.y;
-  const Geom gm = problem_geom(p, prob);
-  const int i = blockIdx.x * kRopeWarps + warp;
-  if (i >= gm.n_new) return;
-  const int32_t ps = pos[p.problems ? gm.new_row + i : i];
-  float cs[4], sn[4];
-#pragma unroll
-  for (int t = 0; t < 4; ++t) rope_sincos(ps, inv_freq[4 * sub + t], sn[t], cs[t]);
-  const int64_t row = gm.new_row + i;
+  const int sub = lane % LPH, hoff = lane / LPH;
   const int n_vec = p.h_q + p.h_kv;
-  for (int base = 0; base < n_vec; base += HPP * 4) {
-    uint2 x1[4], x2[4];
-    int hv[4];
+  const int64_t total = static_cast<int64_t>(n_prob) * rows_per_problem_max;
+  for (int64_t it = static_cast<int64_t>(blockIdx.x) * kRopeWarps + warp; it < total;
+       it += static_cast<int64_t>(gridDim.x) * kRopeWarps) {
+    const int prob = static_cast<int>(it / rows_per_problem_max);
+    const int i = static_cast<int>(it - static_cast<int64_t>(prob) * rows_per_problem_max);
+    const Geom gm = problem_geom(p, prob);
+    if (i >= gm.n_new) continue;
+    // each pair's angle once per row (a lane takes pairs lane, lane + 32), shared through shared memory
+    const int32_t ps = pos[p.problems ? gm.new_row + i : i];
+    __syncwarp();
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      hv[u] = base + u * HPP + hoff;
-      if (hv[u] < n_vec) {
-        const __nv_bfloat16* src = hv[u] < p.h_q ? q + (row * p.h_q + hv[u]) * D
-                                                 : k + (row * p.h_kv + (hv[u] - p.h_q)) * D;
-        x1[u] = *reinterpret_cast<const uint2*>(src + 4 * sub);
-        x2[u] = *reinterpret_cast<const uint2*>(src + D / 2 + 4 * sub);
-      }
+    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, inv_freq[t], s_sn[warp][t], s_cs[warp][t]);
+    __syncwarp();
+    float cs0[4], cs1[4], sn0[4], sn1[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      cs0[t] = s_cs[warp][8 * sub + t];
+      cs1[t] = s_cs[warp][8 * sub + 4 + t];
+      sn0[t] = s_sn[warp][8 * sub + t];
+      sn1[t] = s_sn[warp][8 * sub + 4 + t];
     }
+    const int64_t row = gm.new_row + i;
+    for (int h0 = hoff; h0 < n_vec; h0 += 2 * HPP) {
+      uint4 x1[2], x2[2];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (hv[u] >= n_vec) continue;
-      uint2 y1, y2;
-      rope_rotate4(x1[u], x2[u], cs, sn, y1, y2);
-      __nv_bfloat16* dst;
-      if (hv[u] < p.h_q) {
-        const int g = hv[u] / p.grp, hl = hv[u] - g * p.grp;
-        const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
-                                static_cast<int64_t>(i) * p.grp + hl;
-        dst = qhat + dst_row * D;
-      } else {
-        dst = khat + (row * p.h_kv + (hv[u] - p.h_q)) * D;
+      for (int u = 0; u < 2; ++u) {
+        const int h = h0 + u * HPP;
+        if (h < n_vec) {
+          const __nv_bfloat16* src = h < p.h_q ? q + (row * p.h_q + h) * D : k + (row * p.h_kv + (h - p.h_q)) * D;
+          x1[u] = *reinterpret_cast<const uint4*>(src + 8 * sub);
+          x2[u] = *reinterpret_cast<const uint4*>(src + D / 2 + 8 * sub);
+        }
       }
-      *reinterpret_cast<uint2*>(dst + 4 * sub) = y1;
-      *reinterpret_cast<uint2*>(dst + D / 2 + 4 * sub) = y2;
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int h = h0 + u * HPP;
+        if (h >= n_vec) continue;
+        uint2 ya, yb, yc, yd;
+        rope_rotate4(make_uint2(x1[u].x, x1[u].y), make_uint2(x2[u].x, x2[u].y), cs0, sn0, ya, yb);
+        rope_rotate4(make_uint2(x1[u].z, x1[u].w), make_uint2(x2[u].z, x2[u].w), cs1, sn1, yc, yd);
+        __nv_bfloat16* dst;
+        if (h < p.h_q) {
+          const int g = h / p.grp, hl = h - g * p.grp;
+          const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
+                                  static_cast<int64_t>(i) * p.grp + hl;
+          dst = qhat + dst_row * D;
+        } else {
+          dst = khat + (row * p.h_kv + (h - p.h_q)) * D;
+        }
+        *reinterpret_cast<uint4*>(dst + 8 * sub) = make_uint4(ya.x, ya.y, yc.x, yc.y);
+        *reinterpret_cast<uint4*>(dst + D / 2 + 8 * sub) = make_uint4(yb.x, yb.y, yd.x, yd.y);
+      }
     }
   }
 }
@@ -777,10 +793,12 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.wait_ns = wait_limit_ns();
   const int n_prob = batch_or_np;
   {
-    dim3 grid((max_n_new + kRopeWarps - 1) / kRopeWarps, n_prob);
+    const int64_t items = static_cast<int64_t>(n_prob) * max_n_new;
+    // persistent: three CTAs per SM at the kernel's register count
+    const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, 3ll * num_sms()));
     rope_pack_kernel<D><<<grid, kRopeWarps * 32, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
                                                           static_cast<const __nv_bfloat16*>(k_new), pos, p,
-                                                          rope_theta, max_n_new, qhat, khat);
+                                                          rope_theta, max_n_new, n_prob, qhat, khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK) return s;
   }
