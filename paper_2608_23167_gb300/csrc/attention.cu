@@ -31,35 +31,16 @@
 #include <atomic>
 #include <mutex>
 
-#include "common.cuh"
+#include "attn_common.cuh"
 #include "rope.cuh"
-#include "sm100_ptx.cuh"
 #include "tmem_io.cuh"
 
 namespace ssm {
 namespace {
 
-constexpr int kBM = 128;            // query rows per tile (tcgen05 M)
-constexpr int kBN = 128;            // keys per tile (tcgen05 N of QK^T, K of PV)
-constexpr int kSub = 32;            // rows per TMA sub-box of a key tile
-constexpr int kAttnThreads = 384;   // warpgroup 0: TMA Q/K (warp 0), MMA (warp 1), TMA V (warp 2); warpgroups 1, 2: slots A, B
-// Register split: the kernel is launched with kLaunchRegs per thread (checked on the host);
-// warpgroup 0 gives back down to kCtrlRegs and the two softmax warpgroups grow to
-// kSoftmaxRegs: 128 * (168 - 72) = 256 * (216 - 168), so the split adds up exactly.
-constexpr int kLaunchRegs = 168;
-constexpr int kCtrlRegs = 72;
-constexpr int kSoftmaxRegs = 216;
-static_assert(128 * (kLaunchRegs - kCtrlRegs) >= 256 * (kSoftmaxRegs - kLaunchRegs), "register split");
-static_assert(kAttnThreads * kLaunchRegs <= 65536, "launch registers");
-constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
 constexpr int kKStages = 2;
 constexpr int kVStages = 3;
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kRescaleLog2 = 8.0f;  // rescale O only when the max grows by > 2^8
-constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kOCol = 256;       // O of slot X at 256 + X * D; S (and P) of slot X at X * 128
-constexpr uint64_t kDrainNs = 200000000ull;
 
 enum Bar {
   Q_FULL = 0,
@@ -90,47 +71,6 @@ struct Layout {
   static constexpr int ALLOC = BYTES + 1024;          // slack to align the base to 1024 B
   static_assert(ALLOC <= 232448, "shared memory budget");
 };
-
-struct AttnParams {
-  const ssm_attn_problem* problems;  // null: uniform batch
-  int32_t n_new_u, n_cache_u;
-  int32_t h_q, h_kv, grp;
-  int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
-  int32_t units_per_pg;              // query-tile pairs per (problem, kv head)
-  int32_t total_units;
-  float scale_log2;                  // softmax scale * log2(e)
-  __nv_bfloat16* out;
-  float* lse;
-  unsigned* err;
-  uint64_t wait_ns;
-};
-
-struct Geom {
-  int64_t new_row, cache_row;
-  int32_t n_new, n_cache;
-};
-
-__device__ __forceinline__ Geom problem_geom(const AttnParams& p, int prob) {
-  Geom g;
-  if (p.problems) {
-    const ssm_attn_problem q = p.problems[prob];
-    g.new_row = q.new_row;
-    g.cache_row = q.cache_row;
-    g.n_new = q.n_new;
-    g.n_cache = q.n_cache;
-  } else {
-    g.n_new = p.n_new_u;
-    g.n_cache = p.n_cache_u;
-    g.new_row = static_cast<int64_t>(prob) * p.n_new_u;
-    g.cache_row = 0;
-  }
-  return g;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<const uint32_t*>(&h);
-}
 
 // ---------------------------------------------------------------------------
 // RoPE + GQA packing of the new rows
@@ -217,37 +157,6 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
 // ---------------------------------------------------------------------------
 // Attention forward
 // ---------------------------------------------------------------------------
-
-// Valid keys in each 32-row sub-box of key tile j (cache sub-boxes first, then
-// new-row sub-boxes); returns true if all 128 keys of the tile are valid.
-__device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub, const Geom& gm, int (&vcnt)[4]) {
-  bool full = true;
-#pragma unroll
-  for (int s4 = 0; s4 < 4; ++s4) {
-    const int sub = 4 * j + s4;
-    int c;
-    if (sub < n_csub) c = min(kSub, gm.n_cache - sub * kSub);
-    else if (sub - n_csub < n_nsub) c = min(kSub, gm.n_new - (sub - n_csub) * kSub);
-    else c = 0;
-    vcnt[s4] = c;
-    full = full && (c == kSub);
-  }
-  return full;
-}
-
-// Warp-level barrier use by the softmax warps: one lane polls (so 256 threads do
-// not hammer the shared-memory pipe the MMA thread and TMA also use) and the
-// result is broadcast; arrivals are one per warp after the lanes converge.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  bool ok = true;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, limit_ns);
-  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-}
-
-__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
-}
 
 // One work unit: a pair of query tiles of one (problem, kv head).
 struct Unit {
@@ -735,6 +644,10 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, 
   return r == CUDA_SUCCESS;
 }
 
+std::atomic<int> g_attention_variant{SSM_ATTN_AUTO};
+
+int attention_variant() { return g_attention_variant.load(); }
+
 template <int D>
 ssm_status launch_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
                             const void* k_cache, const void* v_cache, bool uniform, int32_t batch_or_np,
@@ -749,33 +662,41 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   auto* qhat = static_cast<__nv_bfloat16*>(workspace);
   auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) +
                                                 align_up(static_cast<size_t>(total_new) * h_q * D * 2, 256));
-  CUtensorMap tq, tkc, tvc, tkn, tvn, tkc128, tvc128, tkn128, tvn128;
+  // which kernel: 128-row query tiles unless key tiles (queries on the MMA N dimension)
+  // are requested and every (problem, kv head) has at most kKtMaxRows query rows
+  const bool kt_fits = D == 128 && static_cast<int64_t>(max_n_new) * grp <= kKtMaxRows;
+  const int variant = attention_variant();
+  if (variant == SSM_ATTN_KEY_TILES && !kt_fits) return SSM_ERR_UNSUPPORTED;
+  const bool use_kt = kt_fits && variant == SSM_ATTN_KEY_TILES;
+  AttnMaps m;
   {
     const uint64_t dq[3] = {static_cast<uint64_t>(D),
                             static_cast<uint64_t>(uniform ? new_rows_per_b * grp : total_new * h_q),
                             static_cast<uint64_t>(uniform ? nb * h_kv : 1)};
     const uint32_t bq[3] = {64, kBM, 1};
-    if (!make_map(&tq, qhat, 3, dq, bq)) return SSM_ERR_CUDA;
+    if (!make_map(&m.q128, qhat, 3, dq, bq)) return SSM_ERR_CUDA;
+    const uint32_t bq96[3] = {64, 96, 1};
+    if (!make_map(&m.q96, qhat, 3, dq, bq96)) return SSM_ERR_CUDA;
     const uint32_t bkv[4] = {64, 1, kSub, 1};
     const uint64_t dn[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
                             static_cast<uint64_t>(new_rows_per_b), static_cast<uint64_t>(nb)};
-    if (!make_map(&tkn, khat, 4, dn, bkv)) return SSM_ERR_CUDA;
-    if (!make_map(&tvn, v_new, 4, dn, bkv)) return SSM_ERR_CUDA;
+    if (!make_map(&m.kn, khat, 4, dn, bkv)) return SSM_ERR_CUDA;
+    if (!make_map(&m.vn, v_new, 4, dn, bkv)) return SSM_ERR_CUDA;
     const uint32_t bkv128[4] = {64, 1, kBN, 1};
-    if (!make_map(&tkn128, khat, 4, dn, bkv128)) return SSM_ERR_CUDA;
-    if (!make_map(&tvn128, v_new, 4, dn, bkv128)) return SSM_ERR_CUDA;
+    if (!make_map(&m.kn128, khat, 4, dn, bkv128)) return SSM_ERR_CUDA;
+    if (!make_map(&m.vn128, v_new, 4, dn, bkv128)) return SSM_ERR_CUDA;
     if (cache_rows_per_b > 0) {
       const uint64_t dc[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
                               static_cast<uint64_t>(cache_rows_per_b), static_cast<uint64_t>(nb)};
-      if (!make_map(&tkc, k_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
-      if (!make_map(&tvc, v_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
-      if (!make_map(&tkc128, k_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
-      if (!make_map(&tvc128, v_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
+      if (!make_map(&m.kc, k_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
+      if (!make_map(&m.vc, v_cache, 4, dc, bkv)) return SSM_ERR_CUDA;
+      if (!make_map(&m.kc128, k_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
+      if (!make_map(&m.vc128, v_cache, 4, dc, bkv128)) return SSM_ERR_CUDA;
     } else {
-      tkc = tkn;  // never read: no problem has cache rows
-      tvc = tvn;
-      tkc128 = tkn128;
-      tvc128 = tvn128;
+      m.kc = m.kn;  // never read: no problem has cache rows
+      m.vc = m.vn;
+      m.kc128 = m.kn128;
+      m.vc128 = m.vn128;
     }
   }
   AttnParams p{};
@@ -801,6 +722,13 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                                                           rope_theta, max_n_new, n_prob, qhat, khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK) return s;
+  }
+  if (use_kt) {
+    p.units_per_pg = 1;
+    const int64_t total_units = static_cast<int64_t>(n_prob) * h_kv;
+    if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
+    p.total_units = static_cast<int32_t>(total_units);
+    return launch_attn_keytile(m, p, static_cast<int>(std::min<int64_t>(total_units, num_sms())), st);
   }
   // the warpgroup register split assumes the compiled register count
   {
@@ -831,7 +759,8 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
   p.total_units = static_cast<int32_t>(total_units);
   const int grid = static_cast<int>(std::min<int64_t>(total_units, num_sms()));
-  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(tq, tkc, tvc, tkn, tvn, tkc128, tvc128, tkn128, tvn128, p);
+  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128, m.kn128,
+                                                           m.vn128, p);
   return launch_status();
 }
 
@@ -852,6 +781,13 @@ ssm_status check_attn(const void* q, const void* k_new, const void* v_new, const
 }  // namespace ssm
 
 extern "C" {
+
+ssm_status ssm_set_attention_variant(int32_t variant) {
+  if (variant != SSM_ATTN_AUTO && variant != SSM_ATTN_QUERY_TILES && variant != SSM_ATTN_KEY_TILES)
+    return SSM_ERR_INVALID_ARG;
+  ssm::g_attention_variant.store(variant);
+  return SSM_OK;
+}
 
 size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv, int32_t head_dim) {
   if (total_new_rows <= 0 || h_q <= 0 || h_kv <= 0 || head_dim <= 0) return 0;

@@ -1,0 +1,123 @@
+// attn_common.cuh -- pieces shared by the two attention forward kernels
+// (attention.cu: 128-row query tiles; attn_keytile.cu: 128-key tiles with the
+// queries on the MMA N dimension): tile constants, the launch parameters, the
+// per-problem geometry, key-tile validity and the warp-level barrier helpers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "common.cuh"
+#include "sm100_ptx.cuh"
+
+namespace ssm {
+
+constexpr int kBM = 128;            // query rows per tile (tcgen05 M) of the query-tile kernel
+constexpr int kBN = 128;            // keys per tile
+constexpr int kSub = 32;            // rows per TMA sub-box of a key tile
+constexpr int kAttnThreads = 384;   // warpgroup 0: TMA Q/K (warp 0), MMA (warp 1), TMA V (warp 2), K/V watcher (warp 3); warpgroups 1, 2: slots A, B
+// Register split: the kernels are launched with kLaunchRegs per thread (checked on the host);
+// warpgroup 0 gives back down to kCtrlRegs and the two softmax warpgroups grow to
+// kSoftmaxRegs: 128 * (168 - 72) = 256 * (216 - 168), so the split adds up exactly.
+constexpr int kLaunchRegs = 168;
+constexpr int kCtrlRegs = 72;
+constexpr int kSoftmaxRegs = 216;
+static_assert(128 * (kLaunchRegs - kCtrlRegs) >= 256 * (kSoftmaxRegs - kLaunchRegs), "register split");
+static_assert(kAttnThreads * kLaunchRegs <= 65536, "launch registers");
+constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizzle panel
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kRescaleLog2 = 8.0f;  // rescale O only when a maximum grows by > 2^8
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kDrainNs = 200000000ull;
+
+struct AttnParams {
+  const ssm_attn_problem* problems;  // null: uniform batch
+  int32_t n_new_u, n_cache_u;
+  int32_t h_q, h_kv, grp;
+  int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
+  int32_t units_per_pg;              // work units per (problem, kv head)
+  int32_t total_units;
+  float scale_log2;                  // softmax scale * log2(e)
+  __nv_bfloat16* out;
+  float* lse;
+  unsigned* err;
+  uint64_t wait_ns;
+};
+
+struct Geom {
+  int64_t new_row, cache_row;
+  int32_t n_new, n_cache;
+};
+
+__device__ __forceinline__ Geom problem_geom(const AttnParams& p, int prob) {
+  Geom g;
+  if (p.problems) {
+    const ssm_attn_problem q = p.problems[prob];
+    g.new_row = q.new_row;
+    g.cache_row = q.cache_row;
+    g.n_new = q.n_new;
+    g.n_cache = q.n_cache;
+  } else {
+    g.n_new = p.n_new_u;
+    g.n_cache = p.n_cache_u;
+    g.new_row = static_cast<int64_t>(prob) * p.n_new_u;
+    g.cache_row = 0;
+  }
+  return g;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Valid keys in each 32-row sub-box of key tile j (cache sub-boxes first, then
+// new-row sub-boxes); returns true if all 128 keys of the tile are valid.
+__device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub, const Geom& gm, int (&vcnt)[4]) {
+  bool full = true;
+#pragma unroll
+  for (int s4 = 0; s4 < 4; ++s4) {
+    const int sub = 4 * j + s4;
+    int c;
+    if (sub < n_csub) c = min(kSub, gm.n_cache - sub * kSub);
+    else if (sub - n_csub < n_nsub) c = min(kSub, gm.n_new - (sub - n_csub) * kSub);
+    else c = 0;
+    vcnt[s4] = c;
+    full = full && (c == kSub);
+  }
+  return full;
+}
+
+// Warp-level barrier use by the softmax warps: one lane polls (so 256 threads do
+// not hammer the shared-memory pipe the MMA thread and TMA also use) and the
+// result is broadcast; arrivals are one per warp after the lanes converge.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, limit_ns);
+  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+}
+
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
+// The tensor maps both kernels read: queries packed by GQA group (boxes of 128
+// and of 96 rows), and the cache / new-row keys and values in 32-row and
+// 128-row boxes.
+struct AttnMaps {
+  CUtensorMap q128, q96, kc, vc, kn, vn, kc128, vc128, kn128, vn128;
+};
+
+// Largest number of rows (query x head-in-group) of one (problem, kv head)
+// the key-tile kernel takes; up to kKtSplitKeysMax rows its two softmax slots
+// share the queries and split the key tiles.
+constexpr int kKtMaxRows = 192;
+constexpr int kKtSplitKeysMax = 128;
+
+// Launches attn_keytile_kernel (head_dim 128) on `grid` CTAs.
+ssm_status launch_attn_keytile(const AttnMaps& maps, const AttnParams& p, int grid, cudaStream_t st);
+
+}  // namespace ssm

@@ -21,13 +21,39 @@ def dev():
     return cuda_or_skip()
 
 
-def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_lse=True):
+@pytest.fixture(params=["auto", "query_tiles", "key_tiles"])
+def variant(request, dev):
+    """Runs a test under each attention kernel (include/ssm.h: ssm_set_attention_variant)."""
+    from paper_2608_23167_gb300 import ssm
+    code = {"auto": ssm.SSM_ATTN_AUTO, "query_tiles": ssm.SSM_ATTN_QUERY_TILES,
+            "key_tiles": ssm.SSM_ATTN_KEY_TILES}[request.param]
+    ssm.ssm_set_attention_variant(code)
+    yield request.param
+    ssm.ssm_set_attention_variant(ssm.SSM_ATTN_AUTO)
+
+
+def _key_tiles_fit(n_new, h_q, h_kv, d):
+    return d == 128 and n_new * (h_q // h_kv) <= 192
+
+
+def _ramp(t: torch.Tensor, top: float) -> torch.Tensor:
+    """Scales row i of [batch, rows, h, d] by 1 + (top - 1) i / rows: later keys score higher,
+    so the running maximum keeps growing past the first key tile (the lazy rescale path)."""
+    n = t.shape[1]
+    f = 1.0 + (top - 1.0) * torch.arange(n, dtype=torch.float32) / max(n, 1)
+    return (t.float() * f[None, :, None, None]).to(torch.bfloat16)
+
+
+def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_lse=True, ramp=0.0):
     from paper_2608_23167_gb300 import ssm
     q = W.draw_normal_bf16((batch, n_new, h_q, d), 1.0, seed)
     k = W.draw_normal_bf16((batch, n_new, h_kv, d), 1.0, seed + 1)
     v = W.draw_normal_bf16((batch, n_new, h_kv, d), 1.0, seed + 2)
     kc = W.draw_normal_bf16((batch, n_cache, h_kv, d), 1.0, seed + 3) if n_cache else None
     vc = W.draw_normal_bf16((batch, n_cache, h_kv, d), 1.0, seed + 4) if n_cache else None
+    if ramp and kc is not None:
+        kc = _ramp(kc, ramp)
+        k = (k.float() * ramp).to(torch.bfloat16)  # the new keys come after the cache: the largest
     if pos is None:
         g = torch.Generator().manual_seed(seed + 5)
         pos = (n_cache + torch.randperm(4 * n_new + 7, generator=g)[:n_new]).to(torch.int32)
@@ -42,23 +68,36 @@ def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_l
     return f64(out), ref, (None if lse is None else f64(lse)), ref_lse
 
 
-@pytest.mark.parametrize("batch,n_new,n_cache,h_q,h_kv,d,theta", [
-    (1, 73, 64, 4, 4, 64, 1e4),          # tiny workload (b = 0)
-    (1, 589, 0, 8, 8, 128, 5e5),         # LLaDA no-cache shape (8 of 32 heads), 5 query tiles
-    (2, 132, 512, 14, 2, 128, 1e6),      # Dream GQA, 7 query heads per kv head
-    (2, 101, 512, 8, 8, 128, 5e5),       # serving shape (8 of 32 heads)
-    (1, 1, 0, 2, 1, 64, 1e4),            # a single key
-    (3, 37, 100, 4, 2, 128, 0.0),        # ragged cache (100 = 3*32 + 4), no rotary encoding
-    (1, 200, 1000, 2, 2, 64, 1e4),       # cache and new segments both ragged
-    (1, 129, 31, 4, 4, 128, 5e5),        # one row past a query tile
+@pytest.mark.parametrize("batch,n_new,n_cache,h_q,h_kv,d,theta,ramp", [
+    (1, 73, 64, 4, 4, 64, 1e4, 0),          # tiny workload (b = 0)
+    (1, 589, 0, 8, 8, 128, 5e5, 0),         # LLaDA no-cache shape (8 of 32 heads), 5 query tiles
+    (2, 132, 512, 14, 2, 128, 1e6, 0),      # Dream GQA, 7 query heads per kv head
+    (2, 101, 512, 8, 8, 128, 5e5, 0),       # serving shape (8 of 32 heads); key tiles: keys split, N = 112
+    (1, 1, 0, 2, 1, 64, 1e4, 0),            # a single key
+    (3, 37, 100, 4, 2, 128, 0.0, 0),        # ragged cache (100 = 3*32 + 4), no rotary encoding
+    (1, 200, 1000, 2, 2, 64, 1e4, 0),       # cache and new segments both ragged
+    (1, 129, 31, 4, 4, 128, 5e5, 0),        # one row past a query tile; key tiles: queries split 80 + 64
+    (1, 172, 1024, 4, 4, 128, 5e5, 0),      # long sweep at block 0; key tiles: queries split 96 + 80
+    (1, 96, 65, 4, 2, 128, 1e4, 0),         # GQA, 192 rows: the key-tile maximum, queries split 96 + 96
+    (1, 128, 77, 2, 2, 128, 1e4, 0),        # 128 rows: the largest keys-split unit (N = 128)
+    (2, 16, 300, 2, 1, 128, 1e4, 0),        # 32 rows, N = 32
+    (1, 5, 0, 2, 2, 128, 1e4, 0),           # one key tile: slot B of a keys-split unit has no work, N = 16
+    (1, 150, 900, 2, 2, 128, 0.0, 4.0),     # cache keys ramped x1..x4: maxima grow past the first tile
+    (1, 100, 900, 2, 2, 128, 0.0, 4.0),     # the same with the keys split between the slots
 ])
-def test_attention_matches_oracle(dev, batch, n_new, n_cache, h_q, h_kv, d, theta):
-    out, ref, lse, ref_lse = _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache)
-    assert_attention_close(out, ref, f"b{batch} n{n_new} c{n_cache} h{h_q}/{h_kv} d{d}")
+def test_attention_matches_oracle(dev, variant, batch, n_new, n_cache, h_q, h_kv, d, theta, ramp):
+    from paper_2608_23167_gb300 import ssm
+    if variant == "key_tiles" and not _key_tiles_fit(n_new, h_q, h_kv, d):
+        with pytest.raises(ssm.SSMError) as e:
+            _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache, ramp=ramp)
+        assert e.value.status == ssm.SSM_ERR_UNSUPPORTED
+        return
+    out, ref, lse, ref_lse = _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache, ramp=ramp)
+    assert_attention_close(out, ref, f"{variant} b{batch} n{n_new} c{n_cache} h{h_q}/{h_kv} d{d}")
     assert np.abs(lse - ref_lse).max() <= 2e-2
 
 
-def test_attention_full_workloads_sampled(dev):
+def test_attention_full_workloads_sampled(dev, variant):
     """Full-size serving and Dream launches; the oracle checks a sample of heads."""
     from paper_2608_23167_gb300 import ssm
     for name in ("serve", "dream"):
@@ -73,6 +112,8 @@ def test_attention_full_workloads_sampled(dev):
         kc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 34)
         vc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 35)
         o = torch.empty((w.batch, n_new, w.h_q, w.head_dim), dtype=torch.bfloat16, device=dev)
+        if variant == "key_tiles" and not _key_tiles_fit(n_new, w.h_q, w.h_kv, w.head_dim):
+            continue
         ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), o, w.rope_theta)
         torch.cuda.synchronize()
         check_device_error()
@@ -86,7 +127,7 @@ def test_attention_full_workloads_sampled(dev):
             assert_attention_close(f64(o[b:b + 1, :, hs]), ref, f"{name} batch {b}")
 
 
-def test_attention_varlen_block_sweep(dev):
+def test_attention_varlen_block_sweep(dev, variant):
     """The long-sequence sweep: every block index 0..63 as one ragged launch over a
     shared prefix cache; the oracle checks several block indices on a few heads."""
     from paper_2608_23167_gb300 import ssm
@@ -125,7 +166,7 @@ def test_attention_varlen_block_sweep(dev):
         assert np.abs(lg[sl][None] - ref_lse).max() <= 2e-2
 
 
-def test_attention_key_permutation_invariance(dev):
+def test_attention_key_permutation_invariance(dev, variant):
     """Permuting the new rows together with their positions permutes the output rows."""
     from paper_2608_23167_gb300 import ssm
     n, c, h, d = 150, 70, 4, 128
