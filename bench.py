@@ -142,6 +142,11 @@ class StepInputs:
         cache = 2 * (self.cache_rows if self.k_cache is not None else 0) * w.h_kv * w.head_dim * e
         return float(qo + kv_new + cache)
 
+    def rope_bytes(self) -> float:
+        """Algorithmic bytes of the RoPE pre-pass: new query and key rows read once, written rotated."""
+        w = self.w
+        return float(2 * self.total_rows * (w.h_q + w.h_kv) * w.head_dim * 2)
+
     def gather_bytes(self) -> float:
         w = self.w
         row = w.hidden * 2
@@ -168,18 +173,22 @@ class StepInputs:
                                         w.topk, w.alpha, self.x, self.pos, prefix_tokens=self.prefix_tokens)
         if ev is not None:
             ev[2].record()
-        ssm.ssm_attention_varlen(self.q, self.k, self.v, self.pos, self.k_cache, self.v_cache, self.attn_tab,
-                                 self.n, self.max_rows, self.max_cache, self.out, w.rope_theta,
-                                 workspace=self.attn_ws)
+        # the attention stage as its two launches (RoPE pre-pass, forward), timed apart
+        args = (self.q, self.k, self.v, self.pos, self.k_cache, self.v_cache, self.attn_tab, self.n,
+                self.max_rows, self.max_cache, self.out, w.rope_theta)
+        ssm.ssm_attention_varlen_rotate(*args, workspace=self.attn_ws)
         if ev is not None:
             ev[3].record()
+        ssm.ssm_attention_varlen_core(*args, workspace=self.attn_ws)
+        if ev is not None:
+            ev[4].record()
         # the threshold rule needs no second-largest probability, so p2 is not requested
         ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=None,
                        threshold=w.threshold, min_commit=1, workspace=self.unmask_ws)
         if ev is not None:
-            ev[4].record()
+            ev[5].record()
 
-    LAUNCHES_PER_STEP = 6   # select, build, rope_pack, attn_fwd, unmask partial, unmask commit
+    LAUNCHES_PER_STEP = 6   # select, build, rope_pack, attn_fwd, unmask stream, unmask commit
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -249,7 +258,7 @@ def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
     for _ in range(warmup):
         inp.step()
     torch.cuda.synchronize()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     if dist_on:
@@ -263,7 +272,7 @@ def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
     if dist_on:
         torch.distributed.barrier()
     total_ms = t_start.elapsed_time(t_end)
-    stages = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])  # ms
+    stages = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs])  # ms
     return total_ms, stages.mean(axis=0)
 
 
@@ -574,9 +583,11 @@ def main():
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
     peaks, peak_src = load_peaks()
-    sel_ms, build_ms, attn_ms, unmask_ms = [float(x) for x in stage_ms]
+    sel_ms, build_ms, rope_ms, core_ms, unmask_ms = [float(x) for x in stage_ms]
+    attn_ms = rope_ms + core_ms
     flops = inp.attn_flops()
-    attn_tflops = flops / (attn_ms * 1e-3) / 1e12
+    attn_tflops = flops / (attn_ms * 1e-3) / 1e12      # the whole attention stage
+    core_tflops = flops / (core_ms * 1e-3) / 1e12      # the forward kernel alone (the dominant kernel)
     tensor_peak = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
     hbm_peak = peaks["hbm_gbs"]
     traffic = None
@@ -584,11 +595,12 @@ def main():
     if os.path.exists(tpath):
         with open(tpath) as f:
             tr = json.load(f)
-        if tr.get("source_digest") == build_lib.source_digest("attention.cu"):
-            traffic = tr.get("dram_bytes_per_launch")
-    roofline = {"bound": "tensor", "achieved": attn_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
-                "frac": attn_tflops / tensor_peak, "traffic": traffic,
-                "kernel": "ssm_attention_varlen (rope_pack_kernel + attn_fwd_kernel)",
+        part = tr.get("parts", {}).get("attn_fwd_kernel")
+        if tr.get("source_digest") == build_lib.source_digest("attention.cu") and part:
+            traffic = (part["dram_read_MB"] + part["dram_write_MB"]) * 1e6
+    roofline = {"bound": "tensor", "achieved": core_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
+                "frac": core_tflops / tensor_peak, "traffic": traffic,
+                "kernel": "attn_fwd_kernel (ssm_attention_varlen_core)",
                 "peak_kind": f"bf16 dense, sustained ({peak_src})",
                 "algorithmic": f"{flops / 1e9:.1f} GFLOP per launch = 4 * heads * head_dim * sum(Nq * Nk)"}
     gb = lambda nbytes, ms: nbytes / (ms * 1e-3) / 1e9  # noqa: E731
@@ -599,6 +611,11 @@ def main():
         "attention_ms": attn_ms, "attention_TFLOPs": attn_tflops,
         "attention_frac_bf16_sustained": attn_tflops / tensor_peak,
         "attention_frac_bf16_burst": attn_tflops / peaks["bf16_tflops"],
+        "attn_rope_ms": rope_ms, "attn_rope_GBps": gb(inp.rope_bytes(), rope_ms),
+        "attn_rope_frac_hbm": gb(inp.rope_bytes(), rope_ms) / hbm_peak,
+        "attn_fwd_ms": core_ms, "attn_fwd_TFLOPs": core_tflops,
+        "attn_fwd_frac_bf16_sustained": core_tflops / tensor_peak,
+        "attn_fwd_frac_bf16_burst": core_tflops / peaks["bf16_tflops"],
         "unmask_ms": unmask_ms, "unmask_GBps": gb(inp.unmask_bytes(), unmask_ms),
         "unmask_frac_hbm": gb(inp.unmask_bytes(), unmask_ms) / hbm_peak,
         "unmask_frac_8TBps_nominal": gb(inp.unmask_bytes(), unmask_ms) / 8000.0,

@@ -234,6 +234,33 @@ ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_
                                 void* out, float* lse, void* workspace, size_t ws_bytes,
                                 ssm_stream_t stream);
 
+/* The two launches ssm_attention_varlen makes, as separate calls with the same
+ * arguments, for a caller that schedules or times them apart:
+ *   ..._rotate writes the rotated queries (packed by GQA group) and the rotated
+ *              new keys into `workspace` (the RoPE pre-pass; q, k_new, pos and
+ *              the problem table are read, v/cache/out/lse are not touched);
+ *   ..._core   runs the attention forward from that workspace (q, k_new and pos
+ *              are not read again).
+ * ..._core must follow a ..._rotate with the same arguments and workspace, in
+ * stream order; ssm_attention_varlen(args) equals ..._rotate(args) followed by
+ * ..._core(args).  Errors as ssm_attention_varlen. */
+ssm_status ssm_attention_varlen_rotate(const void* q, const void* k_new, const void* v_new,
+                                       const int32_t* pos, const void* k_cache, const void* v_cache,
+                                       int64_t total_new_rows, int64_t total_cache_rows,
+                                       const ssm_attn_problem* problems, int32_t n_problems,
+                                       int32_t max_n_new, int32_t max_n_cache, int32_t h_q,
+                                       int32_t h_kv, int32_t head_dim, float rope_theta, float scale,
+                                       void* out, float* lse, void* workspace, size_t ws_bytes,
+                                       ssm_stream_t stream);
+ssm_status ssm_attention_varlen_core(const void* q, const void* k_new, const void* v_new,
+                                     const int32_t* pos, const void* k_cache, const void* v_cache,
+                                     int64_t total_new_rows, int64_t total_cache_rows,
+                                     const ssm_attn_problem* problems, int32_t n_problems,
+                                     int32_t max_n_new, int32_t max_n_cache, int32_t h_q,
+                                     int32_t h_kv, int32_t head_dim, float rope_theta, float scale,
+                                     void* out, float* lse, void* workspace, size_t ws_bytes,
+                                     ssm_stream_t stream);
+
 /* Which attention forward kernel ssm_attention and ssm_attention_varlen run
  * (process-wide setting; both kernels compute the same function and differ
  * only in how the work is laid on the tensor core):

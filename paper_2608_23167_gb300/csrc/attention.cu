@@ -644,6 +644,9 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, 
   return r == CUDA_SUCCESS;
 }
 
+// The two launches of an attention call: the rotary/packing pre-pass and the forward.
+constexpr int kPartBoth = 0, kPartRotate = 1, kPartCore = 2;
+
 std::atomic<int> g_attention_variant{SSM_ATTN_AUTO};
 
 int attention_variant() { return g_attention_variant.load(); }
@@ -654,7 +657,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                             int64_t new_rows_per_b, int64_t cache_rows_per_b, int32_t max_n_new,
                             const ssm_attn_problem* problems, int32_t h_q, int32_t h_kv,
                             float rope_theta, float scale, void* out, float* lse, void* workspace,
-                            cudaStream_t st) {
+                            cudaStream_t st, int part = kPartBoth) {
   using L = Layout<D>;
   const int grp = h_q / h_kv;
   const int64_t nb = uniform ? batch_or_np : 1;
@@ -713,7 +716,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.err = device_error_word();
   p.wait_ns = wait_limit_ns();
   const int n_prob = batch_or_np;
-  {
+  if (part != kPartCore) {
     const int64_t items = static_cast<int64_t>(n_prob) * max_n_new;
     // persistent: three CTAs per SM at the kernel's register count
     const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, 3ll * num_sms()));
@@ -721,7 +724,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                                                           static_cast<const __nv_bfloat16*>(k_new), pos, p,
                                                           rope_theta, max_n_new, n_prob, qhat, khat);
     const ssm_status s = launch_status();
-    if (s != SSM_OK) return s;
+    if (s != SSM_OK || part == kPartRotate) return s;
   }
   if (use_kt) {
     p.units_per_pg = 1;
@@ -818,7 +821,7 @@ ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, co
                                    nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
 }
 
-ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_new,
+static ssm_status attention_varlen_part(int part, const void* q, const void* k_new, const void* v_new,
                                 const int32_t* pos, const void* k_cache, const void* v_cache,
                                 int64_t total_new_rows, int64_t total_cache_rows,
                                 const ssm_attn_problem* problems, int32_t n_problems,
@@ -841,10 +844,32 @@ ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_
   if (head_dim == 128)
     return ssm::launch_attention<128>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
                                       total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out,
-                                      lse, workspace, st);
+                                      lse, workspace, st, part);
   return ssm::launch_attention<64>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
                                    total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out, lse,
-                                   workspace, st);
+                                   workspace, st, part);
+}
+
+
+#define SSM_VARLEN_PARAMS                                                                                   \
+  const void *q, const void *k_new, const void *v_new, const int32_t *pos, const void *k_cache,            \
+      const void *v_cache, int64_t total_new_rows, int64_t total_cache_rows, const ssm_attn_problem *problems, \
+      int32_t n_problems, int32_t max_n_new, int32_t max_n_cache, int32_t h_q, int32_t h_kv, int32_t head_dim, \
+      float rope_theta, float scale, void *out, float *lse, void *workspace, size_t ws_bytes, ssm_stream_t stream
+#define SSM_VARLEN_ARGS                                                                                     \
+  q, k_new, v_new, pos, k_cache, v_cache, total_new_rows, total_cache_rows, problems, n_problems, max_n_new,  \
+      max_n_cache, h_q, h_kv, head_dim, rope_theta, scale, out, lse, workspace, ws_bytes, stream
+
+ssm_status ssm_attention_varlen(SSM_VARLEN_PARAMS) {
+  return attention_varlen_part(ssm::kPartBoth, SSM_VARLEN_ARGS);
+}
+
+ssm_status ssm_attention_varlen_rotate(SSM_VARLEN_PARAMS) {
+  return attention_varlen_part(ssm::kPartRotate, SSM_VARLEN_ARGS);
+}
+
+ssm_status ssm_attention_varlen_core(SSM_VARLEN_PARAMS) {
+  return attention_varlen_part(ssm::kPartCore, SSM_VARLEN_ARGS);
 }
 
 }  // extern "C"

@@ -78,6 +78,10 @@ def lib() -> ctypes.CDLL:
                                              vp, vp, vp, sz, vp]),
             "ssm_attention_varlen": (ctypes.c_int, [vp, vp, vp, vp, vp, vp, i64, i64, vp, i32, i32, i32, i32,
                                                     i32, i32, f32, f32, vp, vp, vp, sz, vp]),
+            "ssm_attention_varlen_rotate": (ctypes.c_int, [vp, vp, vp, vp, vp, vp, i64, i64, vp, i32, i32, i32,
+                                                           i32, i32, i32, f32, f32, vp, vp, vp, sz, vp]),
+            "ssm_attention_varlen_core": (ctypes.c_int, [vp, vp, vp, vp, vp, vp, i64, i64, vp, i32, i32, i32,
+                                                         i32, i32, i32, f32, f32, vp, vp, vp, sz, vp]),
             "ssm_unmask_workspace_size": (sz, [i32, i32, i64, ctypes.c_int]),
             "ssm_unmask": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32, i32,
                                           vp, vp, vp, vp, vp, sz, vp]),
@@ -100,7 +104,8 @@ def exported_symbols() -> Sequence[str]:
             "ssm_set_attention_variant",
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
-            "ssm_attention_varlen", "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
+            "ssm_attention_varlen", "ssm_attention_varlen_rotate", "ssm_attention_varlen_core",
+            "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
             "ssm_cache_append", "ssm_suffix_topk", "ssm_early_stop"]
 
 
@@ -251,9 +256,8 @@ def attn_problems_tensor(rows, device) -> torch.Tensor:
     return torch.from_numpy(a.view(np.uint8).copy()).to(device)
 
 
-def ssm_attention_varlen(q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems: int, max_n_new: int,
-                         max_n_cache: int, out, rope_theta: float, scale: Optional[float] = None, lse=None,
-                         workspace=None, stream=None):
+def _attention_varlen(fn: str, q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems, max_n_new,
+                      max_n_cache, out, rope_theta, scale, lse, workspace, stream):
     total_new, h_q, d = q.shape
     h_kv = k_new.shape[1]
     total_cache = 0 if k_cache is None else k_cache.shape[0]
@@ -262,10 +266,33 @@ def ssm_attention_varlen(q, k_new, v_new, pos, k_cache, v_cache, problems, n_pro
     need = ssm_attention_workspace_size(total_new, h_q, h_kv, d)
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
-    _check("ssm_attention_varlen", lib().ssm_attention_varlen(
+    _check(fn, getattr(lib(), fn)(
         _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(pos), _ptr(k_cache), _ptr(v_cache), total_new, total_cache,
         _ptr(problems), n_problems, max_n_new, max_n_cache, h_q, h_kv, d, float(rope_theta), float(scale),
         _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def ssm_attention_varlen(q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems: int, max_n_new: int,
+                         max_n_cache: int, out, rope_theta: float, scale: Optional[float] = None, lse=None,
+                         workspace=None, stream=None):
+    _attention_varlen("ssm_attention_varlen", q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems,
+                      max_n_new, max_n_cache, out, rope_theta, scale, lse, workspace, stream)
+
+
+def ssm_attention_varlen_rotate(q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems: int,
+                                max_n_new: int, max_n_cache: int, out, rope_theta: float,
+                                scale: Optional[float] = None, lse=None, workspace=None, stream=None):
+    """The RoPE pre-pass of ssm_attention_varlen alone (writes the workspace)."""
+    _attention_varlen("ssm_attention_varlen_rotate", q, k_new, v_new, pos, k_cache, v_cache, problems,
+                      n_problems, max_n_new, max_n_cache, out, rope_theta, scale, lse, workspace, stream)
+
+
+def ssm_attention_varlen_core(q, k_new, v_new, pos, k_cache, v_cache, problems, n_problems: int,
+                              max_n_new: int, max_n_cache: int, out, rope_theta: float,
+                              scale: Optional[float] = None, lse=None, workspace=None, stream=None):
+    """The attention forward of ssm_attention_varlen alone, from a workspace the rotate call wrote."""
+    _attention_varlen("ssm_attention_varlen_core", q, k_new, v_new, pos, k_cache, v_cache, problems,
+                      n_problems, max_n_new, max_n_cache, out, rope_theta, scale, lse, workspace, stream)
 
 
 # ------------------------------------------------------------------------------ suffix top-k

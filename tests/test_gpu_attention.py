@@ -184,3 +184,36 @@ def test_attention_key_permutation_invariance(dev, variant):
                       pos[perm].contiguous(), kc, vc, o2, 1e4)
     torch.cuda.synchronize()
     assert_attention_close(f64(o2), f64(o1[:, perm]), "permuted")
+
+
+def test_attention_varlen_rotate_then_core_equals_one_call(dev):
+    """ssm_attention_varlen_rotate followed by ssm_attention_varlen_core gives exactly the
+    outputs of ssm_attention_varlen (the same two launches, made as two calls)."""
+    from paper_2608_23167_gb300 import ssm
+    h, d = 4, 128
+    cache_rows = 700
+    kc = W.draw_normal_bf16((cache_rows, h, d), 1.0, 61).to(dev)
+    vc = W.draw_normal_bf16((cache_rows, h, d), 1.0, 62).to(dev)
+    sizes = [(150, 600), (37, 700), (90, 0), (1, 33)]
+    rows, new_row = [], 0
+    for n, c in sizes:
+        rows.append((new_row, 0, n, c))
+        new_row += n
+    q = W.draw_normal_bf16((new_row, h, d), 1.0, 63).to(dev)
+    k = W.draw_normal_bf16((new_row, h, d), 1.0, 64).to(dev)
+    v = W.draw_normal_bf16((new_row, h, d), 1.0, 65).to(dev)
+    pos = (cache_rows + torch.randperm(new_row)).to(torch.int32).to(dev)
+    probs = ssm.attn_problems_tensor(rows, dev)
+    args = (q, k, v, pos, kc, vc, probs, len(rows), max(r[2] for r in rows), max(r[3] for r in rows))
+    o1 = torch.empty_like(q)
+    o2 = torch.empty_like(q)
+    l1 = torch.empty((new_row, h), dtype=torch.float32, device=dev)
+    l2 = torch.empty_like(l1)
+    ssm.ssm_attention_varlen(*args, o1, 5e5, lse=l1)
+    ws = torch.empty(ssm.ssm_attention_workspace_size(new_row, h, h, d), dtype=torch.uint8, device=dev)
+    ssm.ssm_attention_varlen_rotate(*args, o2, 5e5, lse=l2, workspace=ws)
+    ssm.ssm_attention_varlen_core(*args, o2, 5e5, lse=l2, workspace=ws)
+    torch.cuda.synchronize()
+    check_device_error()
+    assert torch.equal(o1, o2)
+    assert torch.equal(l1, l2)
