@@ -621,6 +621,20 @@ def main():
         "unmask_frac_8TBps_nominal": gb(inp.unmask_bytes(), unmask_ms) / 8000.0,
     }
 
+    # The step's roofline: each stage at its own bound (HBM stages at the measured copy bandwidth by their
+    # algorithmic bytes, the attention forward at the sustained bf16 peak by its algorithmic FLOPs; the
+    # selector is launch-latency work and counts as zero), summed over the stages of one batch.
+    floor_ms = {"build": inp.gather_bytes() / (hbm_peak * 1e9) * 1e3,
+                "attn_rope": inp.rope_bytes() / (hbm_peak * 1e9) * 1e3,
+                "attn_fwd": flops / (tensor_peak * 1e12) * 1e3,
+                "unmask": inp.unmask_bytes() / (hbm_peak * 1e9) * 1e3}
+    step_floor_ms = sum(floor_ms.values())
+    step_roofline = {"ms_per_step": step_floor_ms, "value": inp.n / (step_floor_ms * 1e-3), "unit": UNIT,
+                     "frac": (inp.n / (total_ms / args.steps * 1e-3)) / (inp.n / (step_floor_ms * 1e-3)),
+                     "stage_floor_ms": floor_ms,
+                     "how": "sum over stages of algorithmic bytes / measured HBM copy GB/s (build, RoPE pre-pass, "
+                            "unmask) and algorithmic FLOPs / measured sustained bf16 TFLOP/s (attention forward)"}
+
     next_rows = None
     if rank == 0 and not args.no_next:
         next_rows = time_next_rows(inp, attn_ms, dev, hbm_peak, tensor_peak)
@@ -644,7 +658,7 @@ def main():
                        "parallelism": "replicas" if world > 1 else "single GPU",
                        "l2": "inputs larger than L2 (each step reads ~%.0f MB)" % (
                            (inp.gather_bytes() + inp.attn_bytes() + inp.unmask_bytes()) / 1e6)},
-            "roofline": roofline, "stages": stages, "clocks": clk, "e2e": e2e,
+            "roofline": roofline, "step_roofline": step_roofline, "stages": stages, "clocks": clk, "e2e": e2e,
             "cpu_baseline": cpu, "gpu_launches": StepInputs.LAUNCHES_PER_STEP * args.steps,
             "next_rows": next_rows,
         }

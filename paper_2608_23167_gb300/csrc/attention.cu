@@ -204,37 +204,40 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool uniform = p.problems == nullptr;
 
-  if (threadIdx.x == 0) {
-    mbar_init(&bars[Q_FULL], 1);
-    mbar_init(&bars[Q_EMPTY], 1);
+  // No control flow in this kernel depends on the lane: each warp walks its loop
+  // as one converged path and a single lane issues through predicated
+  // instructions (the *_if helpers), so every warp reaches the .sync.aligned
+  // TMEM instructions, tcgen05.dealloc and the CTA barriers whole.
+  const bool leader = lane == 0;
+  if (warp == 0) {
+    mbar_init_if(leader, &bars[Q_FULL], 1);
+    mbar_init_if(leader, &bars[Q_EMPTY], 1);
     for (int s = 0; s < kKStages; ++s) {
-      mbar_init(&bars[K_FULL + s], 1);
-      mbar_init(&bars[K_EMPTY + s], 1);
+      mbar_init_if(leader, &bars[K_FULL + s], 1);
+      mbar_init_if(leader, &bars[K_EMPTY + s], 1);
     }
     for (int s = 0; s < kVStages; ++s) {
-      mbar_init(&bars[V_FULL + s], 1);
-      mbar_init(&bars[V_EMPTY + s], 1);
+      mbar_init_if(leader, &bars[V_FULL + s], 1);
+      mbar_init_if(leader, &bars[V_EMPTY + s], 1);
     }
     for (int x = 0; x < 2; ++x) {
-      mbar_init(&bars[S_FULL + x], 1);
-      mbar_init(&bars[P_FULL + x], 5);   // one arrival per softmax warp, one from the K/V watcher
-      mbar_init(&bars[O_DONE + x], 1);
-      mbar_init(&bars[O_FREE + x], 4);
+      mbar_init_if(leader, &bars[S_FULL + x], 1);
+      mbar_init_if(leader, &bars[P_FULL + x], 5);   // one arrival per softmax warp, one from the K/V watcher
+      mbar_init_if(leader, &bars[O_DONE + x], 1);
+      mbar_init_if(leader, &bars[O_FREE + x], 4);
     }
-    mbar_init(&bars[MERGE_FULL], 4);
-    mbar_init(&bars[DRAIN], 1);
+    mbar_init_if(leader, &bars[MERGE_FULL], 4);
+    mbar_init_if(leader, &bars[DRAIN], 1);
     fence_mbar_init();
-  }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish_alloc_permit();
-  }
-  if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kc);
     tma_prefetch_desc(&tm_vc);
     tma_prefetch_desc(&tm_kn);
     tma_prefetch_desc(&tm_vn);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish_alloc_permit();
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -248,55 +251,55 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       // ------------------------------------------------------------- TMA producers
       // warp 0 loads Q and the K ring, warp 2 the V ring, each at its own pace
       const int half = warp == 2 ? 1 : 0;
-      if (lane == 0) {
-        bool ok = true;
-        int qcount = 0;  // units whose Q was loaded
-        int fills = 0;   // tiles loaded into this ring so far (all units)
-        const int nst = half ? kVStages : kKStages;
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const Unit w = make_unit(p, u);
-          if (!w.valid) continue;
-          if (!half) {
-            if (qcount > 0) ok = mbar_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
-            if (!ok) break;
-            const int nq = w.two ? 2 : 1;
-            mbar_arrive_expect_tx(&bars[Q_FULL], nq * L::TILE);
-            for (int x = 0; x < nq; ++x) {
-              int qy, qz;
-              if (uniform) {
-                qy = (w.qt0 + x) * kBM;
-                qz = w.prob * p.h_kv + w.g;
-              } else {
-                qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
-                     (w.qt0 + x) * kBM;
-                qz = 0;
-              }
-  #pragma unroll
-              for (int pn = 0; pn < NP; ++pn)
-                tma_load_3d(smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy, qz);
+      bool ok = true;
+      int qcount = 0;  // units whose Q was loaded
+      int fills = 0;   // tiles loaded into this ring so far (all units)
+      const int nst = half ? kVStages : kKStages;
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, u);
+        if (!w.valid) continue;
+        if (!half) {
+          if (qcount > 0) ok = warp_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
+          if (!ok) break;
+          const int nq = w.two ? 2 : 1;
+          mbar_arrive_expect_tx_if(leader, &bars[Q_FULL], nq * L::TILE);
+          for (int x = 0; x < nq; ++x) {
+            int qy, qz;
+            if (uniform) {
+              qy = (w.qt0 + x) * kBM;
+              qz = w.prob * p.h_kv + w.g;
+            } else {
+              qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
+                   (w.qt0 + x) * kBM;
+              qz = 0;
             }
-            ++qcount;
+#pragma unroll
+            for (int pn = 0; pn < NP; ++pn)
+              tma_load_3d_if(leader, smem + L::Q + x * L::TILE + pn * kPanel, &tm_q, &bars[Q_FULL], pn * 64, qy,
+                             qz);
           }
-          const int c3 = uniform ? w.prob : 0;
-          for (int jt = 0; jt < w.nt && ok; ++jt) {
-            const int st = fills % nst, fill = fills / nst;
-            if (fill > 0) ok = mbar_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
-            if (!ok) break;
-            uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
-            mbar_arrive_expect_tx(full, L::TILE);
-            uint8_t* dst = smem + (half ? L::V : L::K) + st * L::TILE;
-            const int sub0 = 4 * jt;
-            const bool whole_cache = sub0 + 3 < w.n_csub && (sub0 + 4) * kSub <= w.gm.n_cache;
-            const bool whole_new = sub0 >= w.n_csub && (sub0 - w.n_csub + 4) * kSub <= w.gm.n_new;
-            if (whole_cache || whole_new) {
-              const CUtensorMap* map = whole_cache ? (half ? &tm_vc128 : &tm_kc128) : (half ? &tm_vn128 : &tm_kn128);
-              const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
-                                         : (uniform ? (sub0 - w.n_csub) * kSub
-                                                    : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
-  #pragma unroll
-              for (int pn = 0; pn < NP; ++pn) tma_load_4d(dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
-            } else
-  #pragma unroll
+          ++qcount;
+        }
+        const int c3 = uniform ? w.prob : 0;
+        for (int jt = 0; jt < w.nt && ok; ++jt) {
+          const int st = fills % nst, fill = fills / nst;
+          if (fill > 0) ok = warp_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
+          if (!ok) break;
+          uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
+          mbar_arrive_expect_tx_if(leader, full, L::TILE);
+          uint8_t* dst = smem + (half ? L::V : L::K) + st * L::TILE;
+          const int sub0 = 4 * jt;
+          const bool whole_cache = sub0 + 3 < w.n_csub && (sub0 + 4) * kSub <= w.gm.n_cache;
+          const bool whole_new = sub0 >= w.n_csub && (sub0 - w.n_csub + 4) * kSub <= w.gm.n_new;
+          if (whole_cache || whole_new) {
+            const CUtensorMap* map = whole_cache ? (half ? &tm_vc128 : &tm_kc128) : (half ? &tm_vn128 : &tm_kn128);
+            const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
+                                       : (uniform ? (sub0 - w.n_csub) * kSub
+                                                  : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
+#pragma unroll
+            for (int pn = 0; pn < NP; ++pn) tma_load_4d_if(leader, dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
+          } else {
+#pragma unroll
             for (int sb = 0; sb < 4; ++sb) {
               const int sub = 4 * jt + sb;
               const CUtensorMap* map;
@@ -311,150 +314,149 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
                 map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
                 c2 = p.new_rows_extent;
               }
-  #pragma unroll
+#pragma unroll
               for (int pn = 0; pn < NP; ++pn)
-                tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
+                tma_load_4d_if(leader, dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
             }
-            ++fills;
           }
-        }
-        if (!ok) {
-          record_error(p.err, SSM_ERR_TIMEOUT);
-          // let every copy in flight land before the CTA's shared memory is released:
-          // the newest fill of each stage is the only one that can still be in flight
-          if (!half && qcount > 0) mbar_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
-          for (int i = max(0, fills - nst); i < fills; ++i)
-            mbar_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
+          ++fills;
         }
       }
-      __syncwarp();
+      if (!ok) {
+        record_error(p.err, SSM_ERR_TIMEOUT);
+        // let every copy in flight land before the CTA's shared memory is released:
+        // the newest fill of each stage is the only one that can still be in flight
+        if (!half && qcount > 0) warp_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
+        for (int i = max(0, fills - nst); i < fills; ++i)
+          warp_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
+      }
     } else if (warp == 1) {
       // ------------------------------------------------------------- MMA issuer
-      if (lane == 0) {
-        bool ok = true;
-        // operand descriptors: the per-instruction ones differ only in the start address field
-        const uint64_t dQ = sdesc_sw128(smem_u32(smem + L::Q), 16, 1024);
-        const uint64_t dK = sdesc_sw128(smem_u32(smem + L::K), 16, 1024);
-        const uint64_t dV = sdesc_sw128(smem_u32(smem + L::V), kPanel, 1024);
-        int ucount = 0;            // units processed
-        int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
-        int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const Unit w = make_unit(p, u);
-          if (!w.valid) continue;
-          ok = mbar_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
+      bool ok = true;
+      // operand descriptors: the per-instruction ones differ only in the start address field
+      const uint64_t dQ = sdesc_sw128(smem_u32(smem + L::Q), 16, 1024);
+      const uint64_t dK = sdesc_sw128(smem_u32(smem + L::K), 16, 1024);
+      const uint64_t dV = sdesc_sw128(smem_u32(smem + L::V), kPanel, 1024);
+      int ucount = 0;            // units processed
+      int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
+      int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, u);
+        if (!w.valid) continue;
+        ok = warp_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
+        if (!ok) break;
+        int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
+        int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
+        bool freed0 = false, freed1 = false;
+        // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O
+        auto wait_o_free = [&](int x) -> bool {
+          bool& f = x ? freed1 : freed0;
+          if (f) return true;
+          f = true;
+          return ucount == 0 || warp_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
+        };
+        // O_X += P_X V(j) for slot X's latest job
+        auto issue_pv = [&](int x) -> bool {
+          const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
+          int& pv = x ? pv1 : pv0;
+          if (!wait_o_free(x)) return false;
+          // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
+          if (!warp_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
+          const int vi = vbase + jp;
+          tc_fence_after_sync();
+          const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
+          const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
+          const uint32_t acc0 = k > 0 ? 1u : 0u;
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            umma_bf16_ts_if(leader, d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4),
+                            kIdescPV, kk > 0 ? 1u : acc0);
+          umma_commit_if(leader, &bars[O_DONE + x]);
+          if (!w.two || x == 1) umma_commit_if(leader, &bars[V_EMPTY + vi % kVStages]);
+          ++pv;
+          return true;
+        };
+        const int n_jobs = w.two ? 2 * w.nt : w.nt;
+        for (int t = 0; t < n_jobs && ok; ++t) {
+          const int x = t & 1;
+          const int j = w.two ? (t >> 1) : t;
+          const int ki = kbase + j;
+          if ((x ? kx1 : kx0) > 0)
+            ok = issue_pv(x);
+          else
+            ok = warp_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
           if (!ok) break;
-          int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
-          int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
-          bool freed0 = false, freed1 = false;
-          // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O
-          auto wait_o_free = [&](int x) -> bool {
-            bool& f = x ? freed1 : freed0;
-            if (f) return true;
-            f = true;
-            return ucount == 0 || mbar_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
-          };
-          // O_X += P_X V(j) for slot X's latest job
-          auto issue_pv = [&](int x) -> bool {
-            const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
-            int& pv = x ? pv1 : pv0;
-            if (!wait_o_free(x)) return false;
-            // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
-            if (!mbar_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
-            const int vi = vbase + jp;
-            tc_fence_after_sync();
-            const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
-            const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
-            const uint32_t acc0 = k > 0 ? 1u : 0u;
-  #pragma unroll
-            for (int kk = 0; kk < kBN / 16; ++kk)
-              umma_bf16_ts(d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4), kIdescPV,
-                           kk > 0 ? 1u : acc0);
-            umma_commit(&bars[O_DONE + x]);
-            if (!w.two || x == 1) umma_commit(&bars[V_EMPTY + vi % kVStages]);
-            ++pv;
-            return true;
-          };
-          const int n_jobs = w.two ? 2 * w.nt : w.nt;
-          for (int t = 0; t < n_jobs && ok; ++t) {
-            const int x = t & 1;
-            const int j = w.two ? (t >> 1) : t;
-            const int ki = kbase + j;
-            if ((x ? kx1 : kx0) > 0)
-              ok = issue_pv(x);
-            else
-              ok = mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
-            if (!ok) break;
-            const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
-            const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
-            const uint32_t s_tmem = tmem + x * kBN;
-  #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
-              umma_bf16_ss(s_tmem, qb + off, kb + off, kIdescQK, kk > 0 ? 1u : 0u);
-            }
-            umma_commit(&bars[S_FULL + x]);
-            if (!w.two || x == 1) umma_commit(&bars[K_EMPTY + ki % kKStages]);
-            if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
+          tc_fence_after_sync();
+          const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
+          const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
+          const uint32_t s_tmem = tmem + x * kBN;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
+            umma_bf16_ss_if(leader, s_tmem, qb + off, kb + off, kIdescQK, kk > 0 ? 1u : 0u);
           }
-          if (ok) umma_commit(&bars[Q_EMPTY]);
-          if (ok && kx0 > 0) ok = issue_pv(0);
-          if (ok && kx1 > 0) ok = issue_pv(1);
-          if (ok) ok = wait_o_free(0) && wait_o_free(1);
-          kbase += w.nt;
-          vbase += w.nt;
-          ++ucount;
+          umma_commit_if(leader, &bars[S_FULL + x]);
+          if (!w.two || x == 1) umma_commit_if(leader, &bars[K_EMPTY + ki % kKStages]);
+          if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
         }
-        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
-        // every issued MMA completes before tensor memory is released
-        umma_commit(&bars[DRAIN]);
-        mbar_wait(&bars[DRAIN], 0, kDrainNs);
+        if (ok) umma_commit_if(leader, &bars[Q_EMPTY]);
+        if (ok && kx0 > 0) ok = issue_pv(0);
+        if (ok && kx1 > 0) ok = issue_pv(1);
+        if (ok) ok = wait_o_free(0) && wait_o_free(1);
+        kbase += w.nt;
+        vbase += w.nt;
+        ++ucount;
       }
-      __syncwarp();
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+      // every issued MMA completes before tensor memory is released
+      umma_commit_if(leader, &bars[DRAIN]);
+      warp_wait(&bars[DRAIN], 0, kDrainNs);
     } else {
       // ------------------------------------------------------------- K/V watcher (warp 3)
-      // Every mbarrier test costs the MMA-issuing thread ~150 cycles in which it
+      // Every mbarrier test costs the MMA-issuing warp ~150 cycles in which it
       // issues nothing, so this warp takes the K and V waits off it: it walks the
       // issuer's step order and, for each PV, waits until V of that PV and the K
       // tile of the slot's next QK^T have landed, then adds its arrival to the
       // slot's P_FULL phase.  The issuer then waits for P_FULL alone.  To land in
       // the right phase it first waits for the slot's previous phase to complete.
-      if (lane == 0) {
-        bool ok = true;
-        int kbase = 0;
-        int done0 = 0, done1 = 0;  // P_FULL phases this warp has arrived on, per slot
-        // one arrival for slot x's PV of tile jp, whose slot next reads K tile jk (-1: none)
-        auto vouch = [&](int x, int jp, int jk) -> bool {
-          int& d = x ? done1 : done0;
-          if (d > 0 && !mbar_wait(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
-          const int vi = kbase + jp;
-          if (!mbar_wait(&bars[V_FULL + vi % kVStages], (vi / kVStages) & 1, p.wait_ns)) return false;
-          if (jk >= 0) {
-            const int ki = kbase + jk;
-            if (!mbar_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns)) return false;
-          }
-          mbar_arrive(&bars[P_FULL + x]);
-          ++d;
-          return true;
-        };
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const Unit w = make_unit(p, u);
-          if (!w.valid) continue;
-          int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
-          const int n_jobs = w.two ? 2 * w.nt : w.nt;
-          for (int t = 0; t < n_jobs && ok; ++t) {
-            const int x = t & 1;
-            const int j = w.two ? (t >> 1) : t;
-            if ((x ? kx1 : kx0) > 0) ok = vouch(x, x ? jlast1 : jlast0, j);
-            if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
-          }
-          if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
-          if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
-          kbase += w.nt;
+      // Tiles are confirmed strictly in ring order: a parity wait on fill f of a
+      // stage is exact only once fill f-1 of that stage has been seen to land, and
+      // with split keys a slot's next K tile is two fills ahead of its previous one.
+      bool ok = true;
+      int kbase = 0;
+      int done0 = 0, done1 = 0;  // P_FULL phases this warp has arrived on, per slot
+      int kconf = 0, vconf = 0;  // K / V tiles (all units) confirmed landed, in order
+      auto confirm = [&](int full0, int nst, int& conf, int upto) -> bool {
+        for (; conf <= upto; ++conf)
+          if (!warp_wait(&bars[full0 + conf % nst], (conf / nst) & 1, p.wait_ns)) return false;
+        return true;
+      };
+      // one arrival for slot x's PV of tile jp, whose slot next reads K tile jk (-1: none)
+      auto vouch = [&](int x, int jp, int jk) -> bool {
+        int& d = x ? done1 : done0;
+        if (d > 0 && !warp_wait(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
+        if (!confirm(V_FULL, kVStages, vconf, kbase + jp)) return false;
+        if (jk >= 0 && !confirm(K_FULL, kKStages, kconf, kbase + jk)) return false;
+        mbar_arrive_if(leader, &bars[P_FULL + x]);
+        ++d;
+        return true;
+      };
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, u);
+        if (!w.valid) continue;
+        int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
+        const int n_jobs = w.two ? 2 * w.nt : w.nt;
+        for (int t = 0; t < n_jobs && ok; ++t) {
+          const int x = t & 1;
+          const int j = w.two ? (t >> 1) : t;
+          if ((x ? kx1 : kx0) > 0) ok = vouch(x, x ? jlast1 : jlast0, j);
+          if (x) { jlast1 = j; ++kx1; } else { jlast0 = j; ++kx0; }
         }
-        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+        if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
+        if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
+        kbase += w.nt;
       }
-      __syncwarp();
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
     }
   } else {
     // ------------------------------------------------------------- softmax slots (warps 4..11, warpgroups 1 and 2)
@@ -498,7 +500,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const float m_new = fmaxf(m_run, mx * p.scale_log2);
         const bool need = m_new > m_run + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
-          const float alpha = need ? ex2_approx(m_run - m_new) : 1.f;
+          // branch-free per row (selects only): the warp stays converged for the TMEM accesses
+          const float alpha = ex2_approx(need ? m_run - m_new : 0.f);
           if (k > 0) {
             // the previous PV of this slot completed before this S tile was committed
             ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
@@ -513,10 +516,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
               tmem_st_x32(tO + ch * 32, o);
             }
           }
-          if (need) {
-            l_run *= alpha;
-            m_run = m_new;
-          }
+          l_run *= alpha;
+          m_run = need ? m_new : m_run;
         }
         // p = 2^(s * scale * log2 e - m): packed pair FMA, two MUFU ex2, packed pair sums
         const float neg = -m_run, sc = p.scale_log2;
@@ -564,8 +565,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const int qi = pr / p.grp;
         const int h = w.g * p.grp + (pr - qi * p.grp);
         const float m = fmaxf(m_run, mB);
-        const float a = (l_run > 0.f) ? ex2_approx(m_run - m) : 0.f;
-        const float b = (lB > 0.f) ? ex2_approx(mB - m) : 0.f;
+        const float ea = ex2_approx(m_run - m), eb = ex2_approx(mB - m);
+        const float a = (l_run > 0.f) ? ea : 0.f;
+        const float b = (lB > 0.f) ? eb : 0.f;
         const float lsum = a * l_run + b * lB;
         const float inv = 1.f / lsum;
         const float ca = a * inv, cb = b * inv;
@@ -577,20 +579,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           float f[32];
 #pragma unroll
           for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[c]) * ca;
-          if (!w.two && lB > 0.f) {
+          if (!w.two && w.nt >= 2) {  // warp-uniform; cb = 0 for a row slot B gave no weight
             tmem_ld_x32(tOB + ch * 32, o);
 #pragma unroll
             for (int c = 0; c < 32; ++c) f[c] = fmaf(__uint_as_float(o[c]), cb, f[c]);
           }
-          if (valid) {
-            uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+          uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
 #pragma unroll
-            for (int v = 0; v < 4; ++v)
-              d4[v] = make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
-                                 pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7]));
-          }
+          for (int v = 0; v < 4; ++v)
+            st_global_v4_pred(d4 + v,
+                              make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
+                                         pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7])),
+                              valid);
         }
-        if (valid && p.lse) p.lse[(w.gm.new_row + qi) * p.h_q + h] = (m + log2f(lsum)) * kLn2;
+        if (p.lse) st_global_f32_pred(p.lse + (w.gm.new_row + qi) * p.h_q + h, (m + log2f(lsum)) * kLn2, valid);
         // this slot's O (and, with split keys, slot B's O too) may now be overwritten
         tc_fence_before_sync();
         warp_arrive(&bars[O_FREE + x]);

@@ -90,18 +90,25 @@ __device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub,
   return full;
 }
 
-// Warp-level barrier use by the softmax warps: one lane polls (so 256 threads do
-// not hammer the shared-memory pipe the MMA thread and TMA also use) and the
-// result is broadcast; arrivals are one per warp after the lanes converge.
+// Warp-level barrier use by the softmax warps.  Nothing here branches on the lane:
+// tcgen05.ld/st are .sync.aligned, so the warp must still be one converged path when
+// it reaches them, and a lane-0-only poll leaves lane 0 on a path of its own that
+// warp-synchronous intrinsics (shuffles, __syncwarp) wait for but do not merge (a
+// TMEM load issued that way ended a kernel with an unspecified launch failure).
+// So every lane polls the barrier and the loop is steered by warp votes, and the
+// single arrival of a warp is a predicated instruction rather than a branch.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  bool ok = true;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, limit_ns);
-  return __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+  if (__all_sync(0xffffffffu, mbar_test_wait(bar, parity))) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+    if (__any_sync(0xffffffffu, global_timer_ns() - t0 > limit_ns)) return false;
+  }
 }
 
 __device__ __forceinline__ void warp_arrive(uint64_t* bar) {
   __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+  mbar_arrive_if((threadIdx.x & 31) == 0, bar);
 }
 
 // The tensor maps both kernels read: queries packed by GQA group (boxes of 128

@@ -159,29 +159,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool uniform = p.problems == nullptr;
 
-  if (threadIdx.x == 0) {
-    mbar_init(&bars[KT_Q_FULL], 1);
-    mbar_init(&bars[KT_Q_EMPTY], 1);
+  // No control flow here depends on the lane: each control warp walks its loop as one
+  // converged path and lane 0 issues through predicated instructions (the *_if helpers).
+  const bool leader = lane == 0;
+  if (warp == 0) {
+    mbar_init_if(leader, &bars[KT_Q_FULL], 1);
+    mbar_init_if(leader, &bars[KT_Q_EMPTY], 1);
     for (int s = 0; s < kKtStages; ++s) {
-      mbar_init(&bars[KT_K_FULL + s], 1);
-      mbar_init(&bars[KT_K_EMPTY + s], 1);
-      mbar_init(&bars[KT_V_FULL + s], 1);
-      mbar_init(&bars[KT_V_EMPTY + s], 1);
+      mbar_init_if(leader, &bars[KT_K_FULL + s], 1);
+      mbar_init_if(leader, &bars[KT_K_EMPTY + s], 1);
+      mbar_init_if(leader, &bars[KT_V_FULL + s], 1);
+      mbar_init_if(leader, &bars[KT_V_EMPTY + s], 1);
     }
     for (int x = 0; x < 2; ++x) {
-      mbar_init(&bars[KT_S_FULL + x], 1);
-      mbar_init(&bars[KT_P_FULL + x], 5);  // one arrival per softmax warp, one from the K/V watcher
-      mbar_init(&bars[KT_O_DONE + x], 1);
-      mbar_init(&bars[KT_O_FREE + x], 4);
+      mbar_init_if(leader, &bars[KT_S_FULL + x], 1);
+      mbar_init_if(leader, &bars[KT_P_FULL + x], 5);  // one arrival per softmax warp, one from the K/V watcher
+      mbar_init_if(leader, &bars[KT_O_DONE + x], 1);
+      mbar_init_if(leader, &bars[KT_O_FREE + x], 4);
     }
-    mbar_init(&bars[KT_DRAIN], 1);
+    mbar_init_if(leader, &bars[KT_DRAIN], 1);
     fence_mbar_init();
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish_alloc_permit();
   }
-  if (warp == 0 && lane == 0) {
+  if (warp == 0) {
     tma_prefetch_desc(&tm_q128);
     tma_prefetch_desc(&tm_q96);
     tma_prefetch_desc(&tm_kc);
@@ -200,253 +203,248 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
       // ------------------------------------------------------------- TMA producers
       // warp 0 loads Q and the K ring, warp 2 the V ring, each at its own pace
       const int half = warp == 2 ? 1 : 0;
-      if (lane == 0) {
-        bool ok = true;
-        int qcount = 0;  // units whose Q was loaded
-        int fills = 0;   // tiles loaded into this ring so far (all units)
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const KtUnit w = make_kt_unit(p, u);
-          if (!w.valid) continue;
-          if (!half) {
-            if (qcount > 0) ok = mbar_wait(&bars[KT_Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
-            if (!ok) break;
-            int qy, qz;
-            if (uniform) {
-              qy = 0;
-              qz = w.prob * p.h_kv + w.g;
-            } else {
-              qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp);
-              qz = 0;
-            }
-            if (w.qs) {
-              // slot A's rows [0, nA) at panel row 0, slot B's [nA, rows) at panel row 96
-              mbar_arrive_expect_tx(&bars[KT_Q_FULL], 2 * 2 * 96 * 128);
+      bool ok = true;
+      int qcount = 0;  // units whose Q was loaded
+      int fills = 0;   // tiles loaded into this ring so far (all units)
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const KtUnit w = make_kt_unit(p, u);
+        if (!w.valid) continue;
+        if (!half) {
+          if (qcount > 0) ok = warp_wait(&bars[KT_Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
+          if (!ok) break;
+          int qy, qz;
+          if (uniform) {
+            qy = 0;
+            qz = w.prob * p.h_kv + w.g;
+          } else {
+            qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp);
+            qz = 0;
+          }
+          if (w.qs) {
+            // slot A's rows [0, nA) at panel row 0, slot B's [nA, rows) at panel row 96
+            mbar_arrive_expect_tx_if(leader, &bars[KT_Q_FULL], 2 * 2 * 96 * 128);
 #pragma unroll
-              for (int x = 0; x < 2; ++x)
-#pragma unroll
-                for (int pn = 0; pn < 2; ++pn)
-                  tma_load_3d(smem + L::R + pn * kt_qpanel(true) + x * 96 * 128, &tm_q96, &bars[KT_Q_FULL], pn * 64,
-                              qy + x * w.nA, qz);
-            } else {
-              mbar_arrive_expect_tx(&bars[KT_Q_FULL], 2 * 128 * 128);
+            for (int x = 0; x < 2; ++x)
 #pragma unroll
               for (int pn = 0; pn < 2; ++pn)
-                tma_load_3d(smem + L::R + pn * kt_qpanel(false), &tm_q128, &bars[KT_Q_FULL], pn * 64, qy, qz);
-            }
-            ++qcount;
+                tma_load_3d_if(leader, smem + L::R + pn * kt_qpanel(true) + x * 96 * 128, &tm_q96, &bars[KT_Q_FULL], pn * 64,
+                            qy + x * w.nA, qz);
+          } else {
+            mbar_arrive_expect_tx_if(leader, &bars[KT_Q_FULL], 2 * 128 * 128);
+#pragma unroll
+            for (int pn = 0; pn < 2; ++pn)
+              tma_load_3d_if(leader, smem + L::R + pn * kt_qpanel(false), &tm_q128, &bars[KT_Q_FULL], pn * 64, qy, qz);
           }
-          const int c3 = uniform ? w.prob : 0;
-          for (int jt = 0; jt < w.nt && ok; ++jt) {
-            const int st = fills % kKtStages, fill = fills / kKtStages;
-            if (fill > 0) ok = mbar_wait(&bars[(half ? KT_V_EMPTY : KT_K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
-            if (!ok) break;
-            uint64_t* full = &bars[(half ? KT_V_FULL : KT_K_FULL) + st];
-            mbar_arrive_expect_tx(full, kKtTile);
-            uint8_t* dst = smem + (half ? L::V : L::K) + st * kKtTile;
-            const int sub0 = 4 * jt;
-            const bool whole_cache = sub0 + 3 < w.n_csub && (sub0 + 4) * kSub <= w.gm.n_cache;
-            const bool whole_new = sub0 >= w.n_csub && (sub0 - w.n_csub + 4) * kSub <= w.gm.n_new;
-            if (whole_cache || whole_new) {
-              const CUtensorMap* map = whole_cache ? (half ? &tm_vc128 : &tm_kc128) : (half ? &tm_vn128 : &tm_kn128);
-              const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
-                                         : (uniform ? (sub0 - w.n_csub) * kSub
-                                                    : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
-#pragma unroll
-              for (int pn = 0; pn < 2; ++pn) tma_load_4d(dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
-            } else {
-#pragma unroll
-              for (int sb = 0; sb < 4; ++sb) {
-                const int sub = 4 * jt + sb;
-                const CUtensorMap* map;
-                int c2;
-                if (sub < w.n_csub) {
-                  map = half ? &tm_vc : &tm_kc;
-                  c2 = uniform ? sub * kSub : static_cast<int>(w.gm.cache_row + sub * kSub);
-                } else if (sub - w.n_csub < w.n_nsub) {
-                  map = half ? &tm_vn : &tm_kn;
-                  c2 = uniform ? (sub - w.n_csub) * kSub : static_cast<int>(w.gm.new_row + (sub - w.n_csub) * kSub);
-                } else {
-                  map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
-                  c2 = p.new_rows_extent;
-                }
-#pragma unroll
-                for (int pn = 0; pn < 2; ++pn)
-                  tma_load_4d(dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
-              }
-            }
-            ++fills;
-          }
+          ++qcount;
         }
-        if (!ok) {
-          record_error(p.err, SSM_ERR_TIMEOUT);
-          // let every copy in flight land before the CTA's shared memory is released
-          if (!half && qcount > 0) mbar_wait(&bars[KT_Q_FULL], (qcount - 1) & 1, kDrainNs);
-          for (int i = max(0, fills - kKtStages); i < fills; ++i)
-            mbar_wait(&bars[(half ? KT_V_FULL : KT_K_FULL) + i % kKtStages], (i / kKtStages) & 1, kDrainNs);
+        const int c3 = uniform ? w.prob : 0;
+        for (int jt = 0; jt < w.nt && ok; ++jt) {
+          const int st = fills % kKtStages, fill = fills / kKtStages;
+          if (fill > 0) ok = warp_wait(&bars[(half ? KT_V_EMPTY : KT_K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
+          if (!ok) break;
+          uint64_t* full = &bars[(half ? KT_V_FULL : KT_K_FULL) + st];
+          mbar_arrive_expect_tx_if(leader, full, kKtTile);
+          uint8_t* dst = smem + (half ? L::V : L::K) + st * kKtTile;
+          const int sub0 = 4 * jt;
+          const bool whole_cache = sub0 + 3 < w.n_csub && (sub0 + 4) * kSub <= w.gm.n_cache;
+          const bool whole_new = sub0 >= w.n_csub && (sub0 - w.n_csub + 4) * kSub <= w.gm.n_new;
+          if (whole_cache || whole_new) {
+            const CUtensorMap* map = whole_cache ? (half ? &tm_vc128 : &tm_kc128) : (half ? &tm_vn128 : &tm_kn128);
+            const int c2 = whole_cache ? (uniform ? sub0 * kSub : static_cast<int>(w.gm.cache_row + sub0 * kSub))
+                                       : (uniform ? (sub0 - w.n_csub) * kSub
+                                                  : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
+#pragma unroll
+            for (int pn = 0; pn < 2; ++pn) tma_load_4d_if(leader, dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
+          } else {
+#pragma unroll
+            for (int sb = 0; sb < 4; ++sb) {
+              const int sub = 4 * jt + sb;
+              const CUtensorMap* map;
+              int c2;
+              if (sub < w.n_csub) {
+                map = half ? &tm_vc : &tm_kc;
+                c2 = uniform ? sub * kSub : static_cast<int>(w.gm.cache_row + sub * kSub);
+              } else if (sub - w.n_csub < w.n_nsub) {
+                map = half ? &tm_vn : &tm_kn;
+                c2 = uniform ? (sub - w.n_csub) * kSub : static_cast<int>(w.gm.new_row + (sub - w.n_csub) * kSub);
+              } else {
+                map = half ? &tm_vn : &tm_kn;  // beyond both segments: an out-of-range box reads zeros
+                c2 = p.new_rows_extent;
+              }
+#pragma unroll
+              for (int pn = 0; pn < 2; ++pn)
+                tma_load_4d_if(leader, dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
+            }
+          }
+          ++fills;
         }
       }
-      __syncwarp();
+      if (!ok) {
+        record_error(p.err, SSM_ERR_TIMEOUT);
+        // let every copy in flight land before the CTA's shared memory is released
+        if (!half && qcount > 0) warp_wait(&bars[KT_Q_FULL], (qcount - 1) & 1, kDrainNs);
+        for (int i = max(0, fills - kKtStages); i < fills; ++i)
+          warp_wait(&bars[(half ? KT_V_FULL : KT_K_FULL) + i % kKtStages], (i / kKtStages) & 1, kDrainNs);
+      }
     } else if (warp == 1) {
       // ------------------------------------------------------------- MMA issuer
-      if (lane == 0) {
-        bool ok = true;
-        const uint32_t sK = smem_u32(smem + L::K), sV = smem_u32(smem + L::V), sR = smem_u32(smem + L::R);
-        int ucount = 0;            // units processed
-        int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
-        int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const KtUnit w = make_kt_unit(p, u);
-          if (!w.valid) {
-            if (w.rows > kKtMaxRows) record_error(p.err, SSM_ERR_SHAPE);
-            continue;
-          }
-          ok = mbar_wait(&bars[KT_Q_FULL], ucount & 1, p.wait_ns);
-          if (!ok) break;
-          const bool qs = w.qs;
-          uint32_t id_qk[2], id_pv[2], qb[2], pb[2];
-#pragma unroll
-          for (int x = 0; x < 2; ++x) {
-            const int n = x ? w.nB : w.nA;
-            id_qk[x] = idesc_bf16_f32(128, n, false, false);  // S^T = K Q^T: both K-major
-            id_pv[x] = idesc_bf16_f32(128, n, true, true);    // O^T += V^T P^T: both MN-major
-            qb[x] = sR + (qs ? x * 96 * 128 : 0);
-            pb[x] = sR + kt_pt(qs, x);
-          }
-          const int qpan = kt_qpanel(qs);
-          int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
-          int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest S^T
-          bool freed0 = false, freed1 = false;
-          // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O^T
-          auto wait_o_free = [&](int x) -> bool {
-            bool& f = x ? freed1 : freed0;
-            if (f) return true;
-            f = true;
-            return ucount == 0 || mbar_wait(&bars[KT_O_FREE + x], (ucount - 1) & 1, p.wait_ns);
-          };
-          // O^T_X += V^T(j) P^T_X for slot X's latest job
-          auto issue_pv = [&](int x) -> bool {
-            const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
-            int& pv = x ? pv1 : pv0;
-            if (!wait_o_free(x)) return false;
-            // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
-            if (!mbar_wait(&bars[KT_P_FULL + x], pv & 1, p.wait_ns)) return false;
-            const int vi = vbase + jp;
-            tc_fence_after_sync();
-            const uint32_t vaddr = sV + (vi % kKtStages) * kKtTile;
-            const uint32_t d_tmem = tmem + kKtOCol + x * 128;
-#pragma unroll
-            for (int kk = 0; kk < kBN / 16; ++kk)
-              umma_bf16_ss(d_tmem, sdesc_sw128(vaddr + kk * 16 * 128, kPanel, 1024),
-                           sdesc_sw32(pb[x] + kk * 16 * 32, 4096, 256), id_pv[x], (kk > 0 || k > 0) ? 1u : 0u);
-            umma_commit(&bars[KT_O_DONE + x]);
-            if (!qs || x == 1) umma_commit(&bars[KT_V_EMPTY + vi % kKtStages]);
-            ++pv;
-            return true;
-          };
-          const int n_jobs = qs ? 2 * w.nt : w.nt;
-          for (int t = 0; t < n_jobs && ok; ++t) {
-            const int x = t & 1;
-            const int j = qs ? (t >> 1) : t;
-            const int ki = kbase + j;
-            if ((x ? kx1 : kx0) > 0)
-              ok = issue_pv(x);
-            else
-              ok = mbar_wait(&bars[KT_K_FULL + ki % kKtStages], (ki / kKtStages) & 1, p.wait_ns);
-            if (!ok) break;
-            const uint32_t kaddr = sK + (ki % kKtStages) * kKtTile;
-            const uint32_t s_tmem = tmem + x * 128;
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
-              const uint32_t qoff = (kk >> 2) * qpan + (kk & 3) * 32;
-              umma_bf16_ss(s_tmem, sdesc_sw128(kaddr + off, 16, 1024), sdesc_sw128(qb[x] + qoff, 16, 1024), id_qk[x],
-                           kk > 0 ? 1u : 0u);
-            }
-            umma_commit(&bars[KT_S_FULL + x]);
-            if (!qs || x == 1) umma_commit(&bars[KT_K_EMPTY + ki % kKtStages]);
-            if (x) {
-              jlast1 = j;
-              ++kx1;
-            } else {
-              jlast0 = j;
-              ++kx0;
-            }
-          }
-          // The next unit's Q is loaded once Q_EMPTY completes.  After a keys-split unit
-          // whose successor splits the queries, that Q overlaps this unit's P^T of slot A,
-          // so Q_EMPTY then waits for the final PV GEMMs too.
-          bool gate = false;
-          if (!qs) {
-            for (int u2 = u + gridDim.x; u2 < p.total_units; u2 += gridDim.x) {
-              const KtUnit w2 = make_kt_unit(p, u2);
-              if (w2.valid) {
-                gate = w2.qs;
-                break;
-              }
-            }
-          }
-          if (ok && !gate) umma_commit(&bars[KT_Q_EMPTY]);
-          if (ok && kx0 > 0) ok = issue_pv(0);
-          if (ok && kx1 > 0) ok = issue_pv(1);
-          if (ok && gate) umma_commit(&bars[KT_Q_EMPTY]);
-          if (ok) ok = wait_o_free(0) && wait_o_free(1);
-          kbase += w.nt;
-          vbase += w.nt;
-          ++ucount;
+      bool ok = true;
+      const uint32_t sK = smem_u32(smem + L::K), sV = smem_u32(smem + L::V), sR = smem_u32(smem + L::R);
+      int ucount = 0;            // units processed
+      int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
+      int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const KtUnit w = make_kt_unit(p, u);
+        if (!w.valid) {
+          if (w.rows > kKtMaxRows) record_error(p.err, SSM_ERR_SHAPE);
+          continue;
         }
-        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
-        // every issued MMA completes before tensor memory is released
-        umma_commit(&bars[KT_DRAIN]);
-        mbar_wait(&bars[KT_DRAIN], 0, kDrainNs);
+        ok = warp_wait(&bars[KT_Q_FULL], ucount & 1, p.wait_ns);
+        if (!ok) break;
+        const bool qs = w.qs;
+        uint32_t id_qk[2], id_pv[2], qb[2], pb[2];
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+          const int n = x ? w.nB : w.nA;
+          id_qk[x] = idesc_bf16_f32(128, n, false, false);  // S^T = K Q^T: both K-major
+          id_pv[x] = idesc_bf16_f32(128, n, true, true);    // O^T += V^T P^T: both MN-major
+          qb[x] = sR + (qs ? x * 96 * 128 : 0);
+          pb[x] = sR + kt_pt(qs, x);
+        }
+        const int qpan = kt_qpanel(qs);
+        int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
+        int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest S^T
+        bool freed0 = false, freed1 = false;
+        // one O_FREE wait per slot and unit: the previous unit's epilogue has read this slot's O^T
+        auto wait_o_free = [&](int x) -> bool {
+          bool& f = x ? freed1 : freed0;
+          if (f) return true;
+          f = true;
+          return ucount == 0 || warp_wait(&bars[KT_O_FREE + x], (ucount - 1) & 1, p.wait_ns);
+        };
+        // O^T_X += V^T(j) P^T_X for slot X's latest job
+        auto issue_pv = [&](int x) -> bool {
+          const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
+          int& pv = x ? pv1 : pv0;
+          if (!wait_o_free(x)) return false;
+          // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
+          if (!warp_wait(&bars[KT_P_FULL + x], pv & 1, p.wait_ns)) return false;
+          const int vi = vbase + jp;
+          tc_fence_after_sync();
+          const uint32_t vaddr = sV + (vi % kKtStages) * kKtTile;
+          const uint32_t d_tmem = tmem + kKtOCol + x * 128;
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            umma_bf16_ss_if(leader, d_tmem, sdesc_sw128(vaddr + kk * 16 * 128, kPanel, 1024),
+                         sdesc_sw32(pb[x] + kk * 16 * 32, 4096, 256), id_pv[x], (kk > 0 || k > 0) ? 1u : 0u);
+          umma_commit_if(leader, &bars[KT_O_DONE + x]);
+          if (!qs || x == 1) umma_commit_if(leader, &bars[KT_V_EMPTY + vi % kKtStages]);
+          ++pv;
+          return true;
+        };
+        const int n_jobs = qs ? 2 * w.nt : w.nt;
+        for (int t = 0; t < n_jobs && ok; ++t) {
+          const int x = t & 1;
+          const int j = qs ? (t >> 1) : t;
+          const int ki = kbase + j;
+          if ((x ? kx1 : kx0) > 0)
+            ok = issue_pv(x);
+          else
+            ok = warp_wait(&bars[KT_K_FULL + ki % kKtStages], (ki / kKtStages) & 1, p.wait_ns);
+          if (!ok) break;
+          const uint32_t kaddr = sK + (ki % kKtStages) * kKtTile;
+          const uint32_t s_tmem = tmem + x * 128;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * kPanel + (kk & 3) * 32;
+            const uint32_t qoff = (kk >> 2) * qpan + (kk & 3) * 32;
+            umma_bf16_ss_if(leader, s_tmem, sdesc_sw128(kaddr + off, 16, 1024), sdesc_sw128(qb[x] + qoff, 16, 1024), id_qk[x],
+                         kk > 0 ? 1u : 0u);
+          }
+          umma_commit_if(leader, &bars[KT_S_FULL + x]);
+          if (!qs || x == 1) umma_commit_if(leader, &bars[KT_K_EMPTY + ki % kKtStages]);
+          if (x) {
+            jlast1 = j;
+            ++kx1;
+          } else {
+            jlast0 = j;
+            ++kx0;
+          }
+        }
+        // The next unit's Q is loaded once Q_EMPTY completes.  After a keys-split unit
+        // whose successor splits the queries, that Q overlaps this unit's P^T of slot A,
+        // so Q_EMPTY then waits for the final PV GEMMs too.
+        bool gate = false;
+        if (!qs) {
+          for (int u2 = u + gridDim.x; u2 < p.total_units; u2 += gridDim.x) {
+            const KtUnit w2 = make_kt_unit(p, u2);
+            if (w2.valid) {
+              gate = w2.qs;
+              break;
+            }
+          }
+        }
+        if (ok && !gate) umma_commit_if(leader, &bars[KT_Q_EMPTY]);
+        if (ok && kx0 > 0) ok = issue_pv(0);
+        if (ok && kx1 > 0) ok = issue_pv(1);
+        if (ok && gate) umma_commit_if(leader, &bars[KT_Q_EMPTY]);
+        if (ok) ok = wait_o_free(0) && wait_o_free(1);
+        kbase += w.nt;
+        vbase += w.nt;
+        ++ucount;
       }
-      __syncwarp();
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+      // every issued MMA completes before tensor memory is released
+      umma_commit_if(leader, &bars[KT_DRAIN]);
+      warp_wait(&bars[KT_DRAIN], 0, kDrainNs);
     } else {
       // ------------------------------------------------------------- K/V watcher (warp 3)
       // Takes the K and V waits off the MMA thread (each mbarrier test costs it
       // issue time): for each PV it waits until that PV's V tile and the K tile
       // of the slot's next S^T have landed, then adds its arrival to the slot's
       // P_FULL phase, after seeing the slot's previous phase complete.
-      if (lane == 0) {
-        bool ok = true;
-        int kbase = 0;
-        int done0 = 0, done1 = 0;
-        auto vouch = [&](int x, int jp, int jk) -> bool {
-          int& d = x ? done1 : done0;
-          if (d > 0 && !mbar_wait(&bars[KT_P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
-          const int vi = kbase + jp;
-          if (!mbar_wait(&bars[KT_V_FULL + vi % kKtStages], (vi / kKtStages) & 1, p.wait_ns)) return false;
-          if (jk >= 0) {
-            const int ki = kbase + jk;
-            if (!mbar_wait(&bars[KT_K_FULL + ki % kKtStages], (ki / kKtStages) & 1, p.wait_ns)) return false;
+      bool ok = true;
+      int kbase = 0;
+      int done0 = 0, done1 = 0;
+      // tiles are confirmed strictly in ring order: a parity wait on fill f of a stage is
+      // exact only once fill f-1 of that stage has been seen to land
+      int kconf = 0, vconf = 0;
+      auto confirm = [&](int full0, int& conf, int upto) -> bool {
+        for (; conf <= upto; ++conf)
+          if (!warp_wait(&bars[full0 + conf % kKtStages], (conf / kKtStages) & 1, p.wait_ns)) return false;
+        return true;
+      };
+      auto vouch = [&](int x, int jp, int jk) -> bool {
+        int& d = x ? done1 : done0;
+        if (d > 0 && !warp_wait(&bars[KT_P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
+        if (!confirm(KT_V_FULL, vconf, kbase + jp)) return false;
+        if (jk >= 0 && !confirm(KT_K_FULL, kconf, kbase + jk)) return false;
+        mbar_arrive_if(leader, &bars[KT_P_FULL + x]);
+        ++d;
+        return true;
+      };
+      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
+        const KtUnit w = make_kt_unit(p, u);
+        if (!w.valid) continue;
+        int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
+        const int n_jobs = w.qs ? 2 * w.nt : w.nt;
+        for (int t = 0; t < n_jobs && ok; ++t) {
+          const int x = t & 1;
+          const int j = w.qs ? (t >> 1) : t;
+          if ((x ? kx1 : kx0) > 0) ok = vouch(x, x ? jlast1 : jlast0, j);
+          if (x) {
+            jlast1 = j;
+            ++kx1;
+          } else {
+            jlast0 = j;
+            ++kx0;
           }
-          mbar_arrive(&bars[KT_P_FULL + x]);
-          ++d;
-          return true;
-        };
-        for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-          const KtUnit w = make_kt_unit(p, u);
-          if (!w.valid) continue;
-          int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
-          const int n_jobs = w.qs ? 2 * w.nt : w.nt;
-          for (int t = 0; t < n_jobs && ok; ++t) {
-            const int x = t & 1;
-            const int j = w.qs ? (t >> 1) : t;
-            if ((x ? kx1 : kx0) > 0) ok = vouch(x, x ? jlast1 : jlast0, j);
-            if (x) {
-              jlast1 = j;
-              ++kx1;
-            } else {
-              jlast0 = j;
-              ++kx0;
-            }
-          }
-          if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
-          if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
-          kbase += w.nt;
         }
-        if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+        if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
+        if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
+        kbase += w.nt;
       }
-      __syncwarp();
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
     }
   } else {
     // ------------------------------------------------------------- softmax slots (warps 4..11)
@@ -520,15 +518,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
               float r[32];
 #pragma unroll
               for (int i = 0; i < 32; ++i) r[i] = __uint_as_float(u[i]);
-              if (!full) {
+              if (!full) {  // per-lane selects, no branch: the warp stays converged
 #pragma unroll
                 for (int kb = 0; kb < 4; ++kb)
-                  if (!kv[kb])
 #pragma unroll
-                    for (int gq = 0; gq < 4; ++gq) {
-                      r[CI(kb, gq, 0)] = -INFINITY;
-                      r[CI(kb, gq, 1)] = -INFINITY;
-                    }
+                  for (int gq = 0; gq < 4; ++gq) {
+                    r[CI(kb, gq, 0)] = kv[kb] ? r[CI(kb, gq, 0)] : -INFINITY;
+                    r[CI(kb, gq, 1)] = kv[kb] ? r[CI(kb, gq, 1)] : -INFINITY;
+                  }
               }
 #pragma unroll
               for (int gq = 0; gq < 4; ++gq) {
@@ -549,8 +546,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
                 fadd2_acc(b0, b1, p[6], p[7]);
                 fadd2_acc(a0, a1, b0, b1);
                 if (redo) {
-                  if (!((addf >> JC(ch, gq, 0)) & 1u)) a0 = 0.f;
-                  if (!((addf >> JC(ch, gq, 1)) & 1u)) a1 = 0.f;
+                  a0 = ((addf >> JC(ch, gq, 0)) & 1u) ? a0 : 0.f;
+                  a1 = ((addf >> JC(ch, gq, 1)) & 1u) ? a1 : 0.f;
                 }
                 fadd2_acc(l[JC(ch, gq, 0)], l[JC(ch, gq, 1)], a0, a1);
               }
@@ -606,15 +603,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
           // the slot's previous PV, complete before this S^T tile was committed) orders the
           // scratch after every earlier use of the buffer
           float* scr = reinterpret_cast<float*>(pt);  // [4][128]
-          if (lane < 4) {
 #pragma unroll
-            for (int ch = 0; ch < 4; ++ch)
-              if (ch < nch)
+          for (int ch = 0; ch < 4; ++ch)
+            if (ch < nch)
 #pragma unroll
-                for (int gq = 0; gq < 4; ++gq)
-                  *reinterpret_cast<float2*>(scr + quarter * 128 + 32 * ch + 8 * gq + cpair) =
-                      make_float2(cm[JC(ch, gq, 0)], cm[JC(ch, gq, 1)]);
-          }
+              for (int gq = 0; gq < 4; ++gq)
+                st_shared_f32x2_if(lane < 4, scr + quarter * 128 + 32 * ch + 8 * gq + cpair, cm[JC(ch, gq, 0)],
+                                   cm[JC(ch, gq, 1)]);
           named_barrier_sync(bar_id, 128);
 #pragma unroll
           for (int ch = 0; ch < 4; ++ch) {
@@ -637,17 +632,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
           }
           // new reference: -m -= increase (quarter 0's lanes 0-3 hold every column between them;
           // the barrier below publishes it before any thread reads nm_s again)
-          if (quarter == 0 && lane < 4) {
 #pragma unroll
-            for (int ch = 0; ch < 4; ++ch)
-              if (ch < nch)
+          for (int ch = 0; ch < 4; ++ch)
+            if (ch < nch)
 #pragma unroll
-                for (int gq = 0; gq < 4; ++gq) {
-                  float2* q2 = reinterpret_cast<float2*>(nm_s + 32 * ch + 8 * gq + cpair);
-                  const float2 o = first ? make_float2(0.f, 0.f) : *q2;
-                  *q2 = make_float2(o.x - cm[JC(ch, gq, 0)], o.y - cm[JC(ch, gq, 1)]);
-                }
-          }
+              for (int gq = 0; gq < 4; ++gq) {
+                float* q2 = nm_s + 32 * ch + 8 * gq + cpair;
+                const float2 o = first ? make_float2(0.f, 0.f) : *reinterpret_cast<const float2*>(q2);
+                st_shared_f32x2_if(quarter == 0 && lane < 4, q2, o.x - cm[JC(ch, gq, 0)], o.y - cm[JC(ch, gq, 1)]);
+              }
           if (!first) {
             addf = 0u;
 #pragma unroll
@@ -656,7 +649,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
                 const bool jump = cm[i] >= 100.f;
                 const float alpha = ex2_approx(-cm[i]);
                 l[i] = jump ? 0.f : l[i] * alpha;
-                if (jump) addf |= 1u << i;
+                addf |= static_cast<uint32_t>(jump) << i;
                 cm[i] = alpha;
               }
             }
@@ -710,29 +703,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
         float* sl = reinterpret_cast<float*>(pt);  // [4][128] column sums per warp
         float* coef = sl + 512;
         long long* roff = reinterpret_cast<long long*>(sl + 640);
-        if (lane < 4) {
 #pragma unroll
-          for (int ch = 0; ch < 4; ++ch)
-            if (ch < nch)
+        for (int ch = 0; ch < 4; ++ch)
+          if (ch < nch)
 #pragma unroll
-              for (int gq = 0; gq < 4; ++gq)
-                *reinterpret_cast<float2*>(sl + quarter * 128 + 32 * ch + 8 * gq + cpair) =
-                    make_float2(l[JC(ch, gq, 0)], l[JC(ch, gq, 1)]);
-        }
+            for (int gq = 0; gq < 4; ++gq)
+              st_shared_f32x2_if(lane < 4, sl + quarter * 128 + 32 * ch + 8 * gq + cpair, l[JC(ch, gq, 0)],
+                                 l[JC(ch, gq, 1)]);
         named_barrier_sync(bar_id, 128);
-        if (r < n) {
+        {
+          // every lane computes (r < 128 stays inside the scratch); only valid rows store
           const float lsum = (sl[r] + sl[128 + r]) + (sl[256 + r] + sl[384 + r]);
           const int pr = x * w.nA + r;  // packed (query, head-in-group) row
-          long long ro = -1;
-          if (pr < w.rows) {
-            const int qi = pr / p.grp;
-            const int h = w.g * p.grp + (pr - qi * p.grp);
-            const int64_t orow = (w.gm.new_row + qi) * p.h_q + h;
-            ro = orow * D;
-            if (p.lse) p.lse[orow] = (log2f(lsum) - nm_s[r]) * kLn2;
-          }
+          const bool valid = r < n && pr < w.rows;
+          const int qi = pr / p.grp;
+          const int h = w.g * p.grp + (pr - qi * p.grp);
+          const int64_t orow = (w.gm.new_row + qi) * p.h_q + h;
+          if (p.lse) st_global_f32_pred(p.lse + orow, (log2f(lsum) - nm_s[r]) * kLn2, valid);
           coef[r] = 1.f / lsum;
-          roff[r] = ro;
+          roff[r] = valid ? orow * D : -1;
         }
         named_barrier_sync(bar_id, 128);
         for (int c0 = 0; c0 < n; c0 += 16) {
@@ -741,7 +730,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
             const long long ro = roff[c0 + c];
-            if (ro >= 0) p.out[ro + r] = __float2bfloat16_rn(__uint_as_float(o[c]) * coef[c0 + c]);
+            st_global_bf16_if(ro >= 0, p.out + ro + r, __float2bfloat16_rn(__uint_as_float(o[c]) * coef[c0 + c]));
           }
         }
         tc_fence_before_sync();
@@ -755,36 +744,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
         float* ca = sl + 1024;
         float* cb = sl + 1152;
         long long* roff = reinterpret_cast<long long*>(sl + 1280);
-        if (lane < 4) {
 #pragma unroll
-          for (int ch = 0; ch < 4; ++ch)
-            if (ch < nch)
+        for (int ch = 0; ch < 4; ++ch)
+          if (ch < nch)
 #pragma unroll
-              for (int gq = 0; gq < 4; ++gq)
-                *reinterpret_cast<float2*>(sl + x * 512 + quarter * 128 + 32 * ch + 8 * gq + cpair) =
-                    make_float2(l[JC(ch, gq, 0)], l[JC(ch, gq, 1)]);
-        }
+            for (int gq = 0; gq < 4; ++gq)
+              st_shared_f32x2_if(lane < 4, sl + x * 512 + quarter * 128 + 32 * ch + 8 * gq + cpair, l[JC(ch, gq, 0)],
+                                 l[JC(ch, gq, 1)]);
         named_barrier_sync(3, 256);
         const bool has_b = w.nt >= 2;  // slot B processed at least one key tile
-        if (x == 0 && r < n) {
+        if (x == 0) {
+          // every lane computes (r < 128 stays inside the scratch); only valid rows store
           const float la = (sl[r] + sl[128 + r]) + (sl[256 + r] + sl[384 + r]);
           const float lb = has_b ? (sl[512 + r] + sl[640 + r]) + (sl[768 + r] + sl[896 + r]) : 0.f;
           const float ma = -m_all[r], mb = -m_all[128 + r];
           const float m = lb > 0.f ? fmaxf(ma, mb) : ma;
-          const float a = ex2_approx(ma - m);
-          const float b = lb > 0.f ? ex2_approx(mb - m) : 0.f;
+          const float ea = ex2_approx(ma - m), eb = ex2_approx(mb - m);
+          const float a = ea;
+          const float b = lb > 0.f ? eb : 0.f;
           const float lsum = a * la + b * lb;
-          long long ro = -1;
-          if (r < w.rows) {
-            const int qi = r / p.grp;
-            const int h = w.g * p.grp + (r - qi * p.grp);
-            const int64_t orow = (w.gm.new_row + qi) * p.h_q + h;
-            ro = orow * D;
-            if (p.lse) p.lse[orow] = (m + log2f(lsum)) * kLn2;
-          }
+          const bool valid = r < n && r < w.rows;
+          const int qi = r / p.grp;
+          const int h = w.g * p.grp + (r - qi * p.grp);
+          const int64_t orow = (w.gm.new_row + qi) * p.h_q + h;
+          if (p.lse) st_global_f32_pred(p.lse + orow, (m + log2f(lsum)) * kLn2, valid);
           ca[r] = a / lsum;
           cb[r] = b / lsum;
-          roff[r] = ro;
+          roff[r] = valid ? orow * D : -1;
         }
         named_barrier_sync(3, 256);
         // slot x writes columns [x n / 2, (x + 1) n / 2)
@@ -796,11 +782,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
             const long long ro = roff[c0 + c];
-            if (ro >= 0) {
-              float v = __uint_as_float(oa[c]) * ca[c0 + c];
-              if (has_b) v = fmaf(__uint_as_float(ob[c]), cb[c0 + c], v);
-              p.out[ro + r] = __float2bfloat16_rn(v);
-            }
+            float v = __uint_as_float(oa[c]) * ca[c0 + c];
+            if (has_b) v = fmaf(__uint_as_float(ob[c]), cb[c0 + c], v);
+            st_global_bf16_if(ro >= 0, p.out + ro + r, __float2bfloat16_rn(v));
           }
         }
         tc_fence_before_sync();

@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cstdint>
 
 namespace ssm {
@@ -31,6 +32,38 @@ __device__ __forceinline__ void fence_mbar_init() {
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// The *_if forms below act only in the threads whose `pred` holds, through a
+// predicate on the instruction rather than a branch: a whole warp can walk a
+// control loop together while one lane issues, and stays one converged path
+// for the warp-collective (.sync.aligned) instructions and CTA barriers after it.
+
+__device__ __forceinline__ void mbar_init_if(bool pred, uint64_t* bar, uint32_t count) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %2, 0;\n\t"
+      "@p mbarrier.init.shared::cta.b64 [%0], %1;\n\t}\n" ::"r"(smem_u32(bar)),
+      "r"(count), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_if(bool pred, uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "@p mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}\n" ::"r"(smem_u32(bar)),
+      "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx_if(bool pred, uint64_t* bar, uint32_t bytes) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %2, 0;\n\t"
+      "@p mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}\n" ::"r"(smem_u32(bar)),
+      "r"(bytes), "r"(static_cast<uint32_t>(pred))
+      : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
@@ -124,6 +157,30 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_3d_if(bool pred, void* dst, const CUtensorMap* map, uint64_t* bar,
+                                               int c0, int c1, int c2) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %6, 0;\n\t"
+      "@p cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];\n\t}\n" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2),
+      "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d_if(bool pred, void* dst, const CUtensorMap* map, uint64_t* bar,
+                                               int c0, int c1, int c2, int c3) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %7, 0;\n\t"
+      "@p cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];\n\t}\n" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
+      "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
 // ---------------------------------------------------------------- tensor memory
 
 // Whole warp: allocates `ncols` TMEM columns (power of two, 32..512) and
@@ -207,6 +264,29 @@ __device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, u
       : "memory");
 }
 
+// The same two, issued only where `pred` holds (the warp's elected lane).
+__device__ __forceinline__ void umma_bf16_ss_if(bool pred, uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                                uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "@q tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_bf16_ts_if(bool pred, uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "setp.ne.b32 q, %5, 0;\n\t"
+      "@q tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
 // Warpgroup register reallocation (all four warps of a warpgroup, converged).
 template <int N>
 __device__ __forceinline__ void setmaxnreg_dec() {
@@ -217,15 +297,57 @@ __device__ __forceinline__ void setmaxnreg_inc() {
   asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
-// Named barrier over `count` threads (a multiple of 32) of the CTA.
+// Global stores guarded by a predicate inside the instruction rather than by a
+// branch: warps that go on to warp-collective TMEM accesses stay on one path.
+__device__ __forceinline__ void st_global_v4_pred(void* ptr, uint4 v, bool pred) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %5, 0;\n\t"
+      "@p st.global.v4.b32 [%0], {%1, %2, %3, %4};\n\t}\n" ::"l"(ptr),
+      "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void st_global_f32_pred(float* ptr, float v, bool pred) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %2, 0;\n\t"
+      "@p st.global.f32 [%0], %1;\n\t}\n" ::"l"(ptr),
+      "f"(v), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+__device__ __forceinline__ void st_global_bf16_if(bool pred, __nv_bfloat16* ptr, __nv_bfloat16 v) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %2, 0;\n\t"
+      "@p st.global.b16 [%0], %1;\n\t}\n" ::"l"(ptr),
+      "h"(*reinterpret_cast<const unsigned short*>(&v)), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+// Shared-memory store of two floats (8-byte aligned), predicated like the above.
+__device__ __forceinline__ void st_shared_f32x2_if(bool pred, float* ptr, float a, float b) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %3, 0;\n\t"
+      "@p st.shared.v2.f32 [%0], {%1, %2};\n\t}\n" ::"r"(smem_u32(ptr)),
+      "f"(a), "f"(b), "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
+// Named barrier over `count` threads (a multiple of 32) of the CTA.  The non-aligned
+// form, after reconverging the warp: callers reach it from lane-divergent code.
 __device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t count) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+  __syncwarp();
+  asm volatile("barrier.cta.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 // Named barrier over `count` threads that also ORs a predicate across them:
 // every participant gets true if any participant passed true.
 __device__ __forceinline__ bool named_barrier_or(uint32_t id, uint32_t count, bool pred) {
   uint32_t r;
+  __syncwarp();
   asm volatile(
       "{\n\t.reg .pred p, q;\n\t"
       "setp.ne.u32 q, %1, 0;\n\t"
@@ -243,6 +365,16 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit_if(bool pred, uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "@p tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}\n" ::"r"(
+          smem_u32(bar)),
+      "r"(static_cast<uint32_t>(pred))
       : "memory");
 }
 

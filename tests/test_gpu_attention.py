@@ -217,3 +217,38 @@ def test_attention_varlen_rotate_then_core_equals_one_call(dev):
     check_device_error()
     assert torch.equal(o1, o2)
     assert torch.equal(l1, l2)
+
+
+def test_attention_varlen_serving_batch(dev):
+    """The serving batch through the ragged entry point: 8 sequences of 101 new rows, each with
+    its own 512-row prefix cache (cache_row = 512 s), 32 heads: every work unit is one query
+    tile whose key tiles the two softmax slots split.  This launch once ended with an
+    unspecified launch failure (a warp reaching a tcgen05.ld before it had reconverged)."""
+    from paper_2608_23167_gb300 import ssm
+    w = W.WORKLOADS["serve"]
+    r, *_ = O.select_suffix(w.prompt, w.gen, w.block, 0, w.local, w.middle, w.tail)
+    n_new = w.block + len(r)
+    p1 = list(range(W.block_start(w, 0), W.block_start(w, 0) + w.block)) + r
+    H, d = w.h_q, w.head_dim
+    rows = [(s * n_new, s * w.prompt, n_new, w.prompt) for s in range(w.batch)]
+    total = w.batch * n_new
+    q = W.draw_normal_bf16((total, H, d), 1.0, 71)
+    k = W.draw_normal_bf16((total, H, d), 1.0, 72)
+    v = W.draw_normal_bf16((total, H, d), 1.0, 73)
+    kc = W.draw_normal_bf16((w.batch * w.prompt, H, d), 1.0, 74)
+    vc = W.draw_normal_bf16((w.batch * w.prompt, H, d), 1.0, 75)
+    pos = torch.tensor(p1 * w.batch, dtype=torch.int32)
+    out = torch.full((total, H, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    for rep in range(3):
+        ssm.ssm_attention_varlen(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev),
+                                 ssm.attn_problems_tensor(rows, dev), w.batch, n_new, w.prompt, out, w.rope_theta)
+        torch.cuda.synchronize()
+        check_device_error()
+    og = f64(out)
+    for s in (0, 3, w.batch - 1):
+        sl = slice(s * n_new, (s + 1) * n_new)
+        cs = slice(s * w.prompt, (s + 1) * w.prompt)
+        hs = [0, H - 1]
+        ref, _ = O.attention(f64(q[None, sl][:, :, hs]), f64(k[None, sl][:, :, hs]), f64(v[None, sl][:, :, hs]),
+                             pos[sl].numpy(), f64(kc[None, cs][:, :, hs]), f64(vc[None, cs][:, :, hs]), w.rope_theta)
+        assert_attention_close(og[sl][None][:, :, hs], ref, f"serve sequence {s}")
