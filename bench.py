@@ -596,7 +596,7 @@ def main():
         with open(tpath) as f:
             tr = json.load(f)
         part = tr.get("parts", {}).get("attn_fwd_kernel")
-        if tr.get("source_digest") == build_lib.source_digest("attention.cu") and part:
+        if tr.get("source_digest") == build_lib.source_digest(*build_lib.ATTENTION_SOURCES) and part:
             traffic = (part["dram_read_MB"] + part["dram_write_MB"]) * 1e6
     roofline = {"bound": "tensor", "achieved": core_tflops, "peak": tensor_peak, "unit": "TFLOP/s",
                 "frac": core_tflops / tensor_peak, "traffic": traffic,

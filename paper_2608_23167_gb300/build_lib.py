@@ -46,10 +46,19 @@ def _digest() -> str:
     return h.hexdigest()
 
 
-def source_digest(name: str) -> str:
-    """sha256 of one kernel source file (ties recorded profiler counters to a kernel version)."""
-    with open(os.path.join(CSRC, name), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()
+# The files the attention forward kernel is compiled from (its translation unit and the
+# headers it includes): a change in any of them is a new kernel version.
+ATTENTION_SOURCES = ("attention.cu", "attn_common.cuh", "sm100_ptx.cuh", "tmem_io.cuh", "rope.cuh", "common.cuh")
+
+
+def source_digest(*names: str) -> str:
+    """sha256 over kernel source files, in the order given (ties recorded profiler counters
+    to a kernel version)."""
+    h = hashlib.sha256()
+    for name in names:
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
