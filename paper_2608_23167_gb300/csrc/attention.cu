@@ -360,7 +360,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
           int& pv = x ? pv1 : pv0;
           if (!wait_o_free(x)) return false;
-          // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
+          // the K/V watcher's share of this phase vouches for V(jp) and this slot's next K tile
           if (!warp_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
           const int vi = vbase + jp;
           tc_fence_after_sync();
@@ -382,7 +382,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           const int j = w.two ? (t >> 1) : t;
           const int ki = kbase + j;
           if ((x ? kx1 : kx0) > 0)
-            ok = issue_pv(x);
+            ok = issue_pv(x);  // the watcher's share of P_FULL vouches for this slot's next K tile too
           else
             ok = warp_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
           if (!ok) break;
@@ -413,30 +413,36 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       warp_wait(&bars[DRAIN], 0, kDrainNs);
     } else {
       // ------------------------------------------------------------- K/V watcher (warp 3)
-      // Every mbarrier test costs the MMA-issuing warp ~150 cycles in which it
-      // issues nothing, so this warp takes the K and V waits off it: it walks the
-      // issuer's step order and, for each PV, waits until V of that PV and the K
-      // tile of the slot's next QK^T have landed, then adds its arrival to the
-      // slot's P_FULL phase.  The issuer then waits for P_FULL alone.  To land in
-      // the right phase it first waits for the slot's previous phase to complete.
-      // Tiles are confirmed strictly in ring order: a parity wait on fill f of a
-      // stage is exact only once fill f-1 of that stage has been seen to land, and
-      // with split keys a slot's next K tile is two fills ahead of its previous one.
+      // Every mbarrier test costs the MMA-issuing warp ~150 cycles in which it issues
+      // nothing, so this warp takes the K and V waits off it: it walks the issuer's step
+      // order and, for each PV, waits until that PV's V tile and the K tile of the slot's
+      // next QK^T have landed, then adds its arrival to the slot's P_FULL phase (after
+      // seeing the slot's previous phase complete, so it never arrives twice in one phase).
+      // The issuer waits for K itself only for a slot's first tile of a unit.  A parity
+      // wait is exact only while the barrier cannot be two phases from the awaited one:
+      // V tiles are confirmed in ring order and each is released only after a PV this
+      // warp vouched for; for K, the fill before the awaited one is known from the slot's
+      // QK^T completions, which this warp observes in order (comment in vouch).
       bool ok = true;
       int kbase = 0;
       int done0 = 0, done1 = 0;  // P_FULL phases this warp has arrived on, per slot
-      int kconf = 0, vconf = 0;  // K / V tiles (all units) confirmed landed, in order
-      auto confirm = [&](int full0, int nst, int& conf, int upto) -> bool {
-        for (; conf <= upto; ++conf)
-          if (!warp_wait(&bars[full0 + conf % nst], (conf / nst) & 1, p.wait_ns)) return false;
-        return true;
-      };
-      // one arrival for slot x's PV of tile jp, whose slot next reads K tile jk (-1: none)
+      int vconf = 0;             // V tiles (all units) confirmed landed, in order
+      // one arrival for slot x's PV of tile jp
       auto vouch = [&](int x, int jp, int jk) -> bool {
         int& d = x ? done1 : done0;
         if (d > 0 && !warp_wait(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
-        if (!confirm(V_FULL, kVStages, vconf, kbase + jp)) return false;
-        if (jk >= 0 && !confirm(K_FULL, kKStages, kconf, kbase + jk)) return false;
+        // slot x's d-th QK^T (on K tile jp) has completed, so tile jp has landed; every S
+        // of each slot is seen here in order, so the fill before any K tile waited for
+        // below is known to have landed (split keys: tile jp itself; both slots on every
+        // tile: tile jp - 1, or the previous unit's last tile), and the fill after it
+        // needs this vouch: each parity wait stays within its two-phase window
+        if (!warp_wait(&bars[S_FULL + x], d & 1, p.wait_ns)) return false;
+        for (; vconf <= kbase + jp; ++vconf)
+          if (!warp_wait(&bars[V_FULL + vconf % kVStages], (vconf / kVStages) & 1, p.wait_ns)) return false;
+        if (jk >= 0) {
+          const int ki = kbase + jk;
+          if (!warp_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns)) return false;
+        }
         mbar_arrive_if(leader, &bars[P_FULL + x]);
         ++d;
         return true;

@@ -327,7 +327,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
           const int jp = x ? jlast1 : jlast0, k = (x ? kx1 : kx0) - 1;
           int& pv = x ? pv1 : pv0;
           if (!wait_o_free(x)) return false;
-          // the K/V watcher's share of this phase vouches for V(jp) and for this slot's next K tile
+          // the K/V watcher's share of this phase vouches for V(jp) and this slot's next K tile
           if (!warp_wait(&bars[KT_P_FULL + x], pv & 1, p.wait_ns)) return false;
           const int vi = vbase + jp;
           tc_fence_after_sync();
@@ -348,7 +348,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
           const int j = qs ? (t >> 1) : t;
           const int ki = kbase + j;
           if ((x ? kx1 : kx0) > 0)
-            ok = issue_pv(x);
+            ok = issue_pv(x);  // the watcher's share of P_FULL vouches for this slot's next K tile too
           else
             ok = warp_wait(&bars[KT_K_FULL + ki % kKtStages], (ki / kKtStages) & 1, p.wait_ns);
           if (!ok) break;
@@ -399,26 +399,31 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
       warp_wait(&bars[KT_DRAIN], 0, kDrainNs);
     } else {
       // ------------------------------------------------------------- K/V watcher (warp 3)
-      // Takes the K and V waits off the MMA thread (each mbarrier test costs it
-      // issue time): for each PV it waits until that PV's V tile and the K tile
-      // of the slot's next S^T have landed, then adds its arrival to the slot's
-      // P_FULL phase, after seeing the slot's previous phase complete.
+      // Takes the K and V waits off the MMA warp (each mbarrier test costs it issue time):
+      // for each PV it waits until that PV's V tile and the K tile of the slot's next S^T
+      // have landed, then adds its arrival to the slot's P_FULL phase, after seeing the
+      // slot's previous phase complete.  V tiles are confirmed in ring order; for K the
+      // fill before the awaited one is known from the slot's S^T completions, observed in
+      // order (the same scheme as attn_fwd_kernel).
       bool ok = true;
       int kbase = 0;
       int done0 = 0, done1 = 0;
-      // tiles are confirmed strictly in ring order: a parity wait on fill f of a stage is
-      // exact only once fill f-1 of that stage has been seen to land
-      int kconf = 0, vconf = 0;
-      auto confirm = [&](int full0, int& conf, int upto) -> bool {
-        for (; conf <= upto; ++conf)
-          if (!warp_wait(&bars[full0 + conf % kKtStages], (conf / kKtStages) & 1, p.wait_ns)) return false;
-        return true;
-      };
+      int vconf = 0;  // V tiles (all units) confirmed landed, in order
       auto vouch = [&](int x, int jp, int jk) -> bool {
         int& d = x ? done1 : done0;
         if (d > 0 && !warp_wait(&bars[KT_P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
-        if (!confirm(KT_V_FULL, vconf, kbase + jp)) return false;
-        if (jk >= 0 && !confirm(KT_K_FULL, kconf, kbase + jk)) return false;
+        // slot x's d-th QK^T (on K tile jp) has completed, so tile jp has landed; every S
+        // of each slot is seen here in order, so the fill before any K tile waited for
+        // below is known to have landed (split keys: tile jp itself; both slots on every
+        // tile: tile jp - 1, or the previous unit's last tile), and the fill after it
+        // needs this vouch: each parity wait stays within its two-phase window
+        if (!warp_wait(&bars[KT_S_FULL + x], d & 1, p.wait_ns)) return false;
+        for (; vconf <= kbase + jp; ++vconf)
+          if (!warp_wait(&bars[KT_V_FULL + vconf % kKtStages], (vconf / kKtStages) & 1, p.wait_ns)) return false;
+        if (jk >= 0) {
+          const int ki = kbase + jk;
+          if (!warp_wait(&bars[KT_K_FULL + ki % kKtStages], (ki / kKtStages) & 1, p.wait_ns)) return false;
+        }
         mbar_arrive_if(leader, &bars[KT_P_FULL + x]);
         ++d;
         return true;
