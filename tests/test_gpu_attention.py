@@ -252,3 +252,59 @@ def test_attention_varlen_serving_batch(dev):
         ref, _ = O.attention(f64(q[None, sl][:, :, hs]), f64(k[None, sl][:, :, hs]), f64(v[None, sl][:, :, hs]),
                              pos[sl].numpy(), f64(kc[None, cs][:, :, hs]), f64(vc[None, cs][:, :, hs]), w.rope_theta)
         assert_attention_close(og[sl][None][:, :, hs], ref, f"serve sequence {s}")
+
+
+@pytest.mark.parametrize("shape", ["llada", "serve"])
+def test_attention_varlen_cold_l2_and_graph_replay(dev, variant, shape):
+    """Pipeline timing edge cases: every launch behind a 256 MB write (cold L2, slow tile loads
+    while the producers run ahead), eagerly and as CUDA-graph replays, with a 0.2 s wait limit so
+    a stuck barrier wait reports SSM_ERR_TIMEOUT quickly; the outputs must equal a warm launch's.
+    Shapes: one 589-row problem without cache (LLaDA: two-query-tile units and a split-key tail
+    unit), and 8 x 101 rows with per-sequence 512-row caches (serving: split-key units only)."""
+    from paper_2608_23167_gb300 import ssm
+    h, d = 32, 128
+    if shape == "llada":
+        sizes, cache_rows = [(589, 0)], 0
+    else:
+        sizes, cache_rows = [(101, 512)] * 8, 8 * 512
+    if variant == "key_tiles" and not _key_tiles_fit(max(n for n, _ in sizes), h, h, d):
+        pytest.skip("shape outside the key-tile kernel")
+    rows, new_row = [], 0
+    for i, (n, c) in enumerate(sizes):
+        rows.append((new_row, i * c, n, c))
+        new_row += n
+    q = W.draw_normal_bf16((new_row, h, d), 1.0, 81).to(dev)
+    k = W.draw_normal_bf16((new_row, h, d), 1.0, 82).to(dev)
+    v = W.draw_normal_bf16((new_row, h, d), 1.0, 83).to(dev)
+    kc = W.draw_normal_bf16((cache_rows, h, d), 1.0, 84).to(dev) if cache_rows else None
+    vc = W.draw_normal_bf16((cache_rows, h, d), 1.0, 85).to(dev) if cache_rows else None
+    pos = torch.arange(new_row, dtype=torch.int32).to(dev) % 1500 + 512
+    probs = ssm.attn_problems_tensor(rows, dev)
+    ws = torch.empty(ssm.ssm_attention_workspace_size(new_row, h, h, d), dtype=torch.uint8, device=dev)
+    args = (q, k, v, pos, kc, vc, probs, len(rows), max(r[2] for r in rows), max(r[3] for r in rows))
+    ref = torch.empty_like(q)
+    ssm.ssm_attention_varlen(*args, ref, 5e5, workspace=ws)
+    torch.cuda.synchronize()
+    check_device_error()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    out = torch.empty_like(q)
+    ssm.ssm_set_wait_limit_ns(200_000_000)
+    try:
+        for i in range(8):
+            flush.fill_(i)
+            ssm.ssm_attention_varlen(*args, out, 5e5, workspace=ws)
+        torch.cuda.synchronize()
+        check_device_error()
+        assert torch.equal(out, ref)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            ssm.ssm_attention_varlen(*args, out, 5e5, workspace=ws)
+        for i in range(8):
+            flush.fill_(i)
+            out.zero_()
+            g.replay()
+        torch.cuda.synchronize()
+        check_device_error()
+        assert torch.equal(out, ref)
+    finally:
+        ssm.ssm_set_wait_limit_ns(0)
