@@ -488,27 +488,65 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         if (!ok) break;
         tc_fence_after_sync();
         uint32_t sr[kBN];
-        tmem_ld_x128(tS, sr);
         int vcnt[4];
-        if (!tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, vcnt)) {
+        const bool full_tile = tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, vcnt);
+        // this row's scores of the tile, keys past a segment end at -inf
+        auto load_s = [&]() {
+          tmem_ld_x128(tS, sr);
+          if (!full_tile) {
 #pragma unroll
-          for (int c = 0; c < kBN; ++c)
-            if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
-        }
-        // row maximum: eight independent chains of 3-input max, then a short tree
-        float mx8[8];
+            for (int c = 0; c < kBN; ++c)
+              if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
+          }
+        };
+        load_s();
+        const float sc = p.scale_log2;
+        // row maximum of the tile's scores: eight independent chains of 3-input max, then a short tree
+        auto row_max = [&]() -> float {
+          float mx8[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) mx8[c] = __uint_as_float(sr[c]);
+          for (int c = 0; c < 8; ++c) mx8[c] = __uint_as_float(sr[c]);
 #pragma unroll
-        for (int c = 8; c < kBN; c += 2)
-          mx8[(c >> 1) & 7] = fmax3(mx8[(c >> 1) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
-        const float mx = fmaxf(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7]));
-        const float m_new = fmaxf(m_run, mx * p.scale_log2);
-        const bool need = m_new > m_run + kRescaleLog2;
-        if (__any_sync(0xffffffffu, need)) {
-          // branch-free per row (selects only): the warp stays converged for the TMEM accesses
-          const float alpha = ex2_approx(need ? m_run - m_new : 0.f);
-          if (k > 0) {
+          for (int c = 8; c < kBN; c += 2)
+            mx8[(c >> 1) & 7] = fmax3(mx8[(c >> 1) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
+          return fmaxf(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(fmax3(mx8[3], mx8[4], mx8[5]), mx8[6], mx8[7]));
+        };
+        // p = 2^(s * scale * log2 e - m) into pk (bf16 pairs): packed pair FMA, two MUFU ex2, packed
+        // pair sums; returns the row's sum of p over the tile
+        uint32_t pk[kBN / 2];
+        auto exp_pass = [&](float m) -> float {
+          const float neg = -m;
+          float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int c = 0; c < kBN / 2; ++c) {
+            float t0, t1;
+            ffma2(t0, t1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), sc, sc, neg, neg);
+            const float a = ex2_approx(t0), b = ex2_approx(t1);
+            fadd2_acc(ra[c & 3], rb[c & 3], a, b);
+            pk[c] = pack_bf16x2(a, b);
+          }
+          return ((ra[0] + rb[0]) + (ra[1] + rb[1])) + ((ra[2] + rb[2]) + (ra[3] + rb[3]));
+        };
+        float lt;
+        if (k == 0) {
+          // the slot's first tile of the unit sets the reference m: its row maximum (finite:
+          // every key tile holds at least one valid key)
+          m_run = row_max() * sc;
+          lt = exp_pass(m_run);
+        } else {
+          // later tiles: exponentials against the current reference without a row maximum.
+          // A tile sum of at most 2^16 bounds every p by 2^16 (far inside fp32 / bf16 range);
+          // a row above it (or inf / NaN) takes the exact path: new m from the row maximum,
+          // O and l rescaled by 2^(m_old - m_new), exponentials again.  Branch-free per row
+          // (selects only): the warp stays converged for the TMEM accesses.
+          lt = exp_pass(m_run);
+          const bool need = !(lt <= kSpecSumMax);
+          if (__any_sync(0xffffffffu, need)) {
+            // S is still in tensor memory (P has not been written over it): load it again
+            // rather than keep the scores live through the exponentials
+            load_s();
+            const float m_new = fmaxf(m_run, row_max() * sc);
+            const float alpha = ex2_approx(need ? m_run - m_new : 0.f);
             // the previous PV of this slot completed before this S tile was committed
             ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
             if (!ok) break;
@@ -521,23 +559,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
               for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
               tmem_st_x32(tO + ch * 32, o);
             }
+            l_run *= alpha;
+            m_run = need ? m_new : m_run;
+            lt = exp_pass(m_run);
           }
-          l_run *= alpha;
-          m_run = need ? m_new : m_run;
         }
-        // p = 2^(s * scale * log2 e - m): packed pair FMA, two MUFU ex2, packed pair sums
-        const float neg = -m_run, sc = p.scale_log2;
-        float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
-        uint32_t pk[kBN / 2];
-#pragma unroll
-        for (int c = 0; c < kBN / 2; ++c) {
-          float t0, t1;
-          ffma2(t0, t1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), sc, sc, neg, neg);
-          const float a = ex2_approx(t0), b = ex2_approx(t1);
-          fadd2_acc(ra[c & 3], rb[c & 3], a, b);
-          pk[c] = pack_bf16x2(a, b);
-        }
-        l_run += ((ra[0] + rb[0]) + (ra[1] + rb[1])) + ((ra[2] + rb[2]) + (ra[3] + rb[3]));
+        l_run += lt;
         // P (bf16) overwrites the first 64 columns of this slot's S; the PV GEMM reads it from there
         tmem_st_x64(tS, pk);
         tc_fence_before_sync();

@@ -29,6 +29,7 @@ constexpr int kPanel = 128 * 128;   // bytes of a 128-row x 64-column bf16 swizz
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleLog2 = 8.0f;  // rescale O only when a maximum grows by > 2^8
+constexpr float kSpecSumMax = 65536.0f;  // a tile's row sum of p above this takes the exact path
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 200000000ull;
 

@@ -84,6 +84,8 @@ def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_l
     (1, 5, 0, 2, 2, 128, 1e4, 0),           # one key tile: slot B of a keys-split unit has no work, N = 16
     (1, 150, 900, 2, 2, 128, 0.0, 4.0),     # cache keys ramped x1..x4: maxima grow past the first tile
     (1, 100, 900, 2, 2, 128, 0.0, 4.0),     # the same with the keys split between the slots
+    (1, 150, 900, 2, 2, 128, 0.0, 16.0),    # x1..x16: later tiles' p reach 2^50 against the first tile's
+    (1, 100, 900, 2, 2, 128, 0.0, 16.0),    #   maximum, so the exact (rescaling) path runs, both layouts
 ])
 def test_attention_matches_oracle(dev, variant, batch, n_new, n_cache, h_q, h_kv, d, theta, ramp):
     from paper_2608_23167_gb300 import ssm
