@@ -78,6 +78,68 @@ struct Layout {
 
 constexpr int kRopeWarps = 8;
 
+// Problem whose new rows contain row r: the last problem starting at or before r
+// (problems of a packable plan start at increasing rows).
+__device__ __forceinline__ int problem_of_row(const ssm_attn_problem* pr, int n_prob, int64_t r) {
+  int lo = 0, hi = n_prob - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (pr[mid].new_row <= r) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// The unit plan of a ragged batch (one warp).  Packed units are used when every problem
+// reads the same cache rows (the same cache_row), the problems' new rows follow one
+// another from row 0 without gaps, and packing needs fewer 128-row query tiles than one
+// problem per unit does.
+__device__ void attn_plan_warp(const AttnParams& p, int n_prob, int64_t total_new, int max_pairs) {
+  const int lane = threadIdx.x & 31;
+  const ssm_attn_problem* pr = p.problems;
+  const int64_t c0 = pr[0].cache_row;
+  bool ok = true;
+  int64_t tiles = 0;
+  for (int b = lane; b < n_prob; b += 32) {
+    const ssm_attn_problem q = pr[b];
+    const int64_t expect = b == 0 ? 0 : pr[b - 1].new_row + pr[b - 1].n_new;
+    ok = ok && q.cache_row == c0 && q.new_row == expect && q.n_new > 0;
+    tiles += (static_cast<int64_t>(q.n_new) * p.grp + kBM - 1) / kBM;
+  }
+  ok = __all_sync(0xffffffffu, ok);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tiles += __shfl_xor_sync(0xffffffffu, tiles, o);
+  const int64_t last_end = pr[n_prob - 1].new_row + pr[n_prob - 1].n_new;
+  const int64_t qrows = total_new * p.grp;
+  const int64_t packed_tiles = (qrows + kBM - 1) / kBM;
+  const int n_pairs = static_cast<int>((qrows + 2 * kBM - 1) / (2 * kBM));
+  const bool packed = ok && last_end == total_new && packed_tiles < tiles && n_pairs <= max_pairs;
+  AttnPlanUnit* units = reinterpret_cast<AttnPlanUnit*>(p.plan + 1);
+  if (packed) {
+    for (int i = lane; i < n_pairs; i += 32) {
+      AttnPlanUnit u;
+      const int64_t p0 = static_cast<int64_t>(i) * 2 * kBM;
+      u.p0 = static_cast<int32_t>(p0);
+      u.rows = static_cast<int32_t>(qrows - p0 < 2 * kBM ? qrows - p0 : 2 * kBM);
+      const int b_lo = problem_of_row(pr, n_prob, p0 / p.grp);
+      const int b_hi = problem_of_row(pr, n_prob, (p0 + u.rows - 1) / p.grp);
+      int c_max = 0;
+      for (int b = b_lo; b <= b_hi; ++b) c_max = max(c_max, pr[b].n_cache);
+      u.c_max = c_max;
+      u.pad = 0;
+      u.nr_lo = pr[b_lo].new_row;
+      u.nr_hi = pr[b_hi].new_row + pr[b_hi].n_new;
+      units[i] = u;
+    }
+  }
+  if (lane == 0) {
+    AttnPlanHdr h{};
+    h.packed = packed ? 1 : 0;
+    h.n_pairs = packed ? n_pairs : 0;
+    h.cache_row = c0;
+    *p.plan = h;
+  }
+}
+
 // Persistent warps over (problem, row) items, item = problem * rows_per_problem_max
 // + row (items past a problem's row count are skipped).  A row's D/2 angles are
 // formed once (two per lane) and shared through shared memory; a lane then owns
@@ -88,7 +150,7 @@ template <int D>
 __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
     const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max, int32_t n_prob,
-    __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
+    int32_t max_pairs, __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
   constexpr int LPH = D / 16;       // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
@@ -96,6 +158,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
   if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (p.plan && blockIdx.x == 0 && warp == 0) attn_plan_warp(p, n_prob, p.new_rows_extent, max_pairs);
   const int sub = lane % LPH, hoff = lane / LPH;
   const int n_vec = p.h_q + p.h_kv;
   const int64_t total = static_cast<int64_t>(n_prob) * rows_per_problem_max;
@@ -120,6 +183,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
       sn1[t] = s_sn[warp][8 * sub + 4 + t];
     }
     const int64_t row = gm.new_row + i;
+    if (p.row_prob && lane == 0) p.row_prob[row] = prob;
     for (int h0 = hoff; h0 < n_vec; h0 += 2 * HPP) {
       uint4 x1[2], x2[2];
 #pragma unroll
@@ -140,9 +204,13 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
         rope_rotate4(make_uint2(x1[u].z, x1[u].w), make_uint2(x2[u].z, x2[u].w), cs1, sn1, yc, yd);
         __nv_bfloat16* dst;
         if (h < p.h_q) {
+          // queries packed by GQA group: a uniform batch per (problem, kv head); a ragged batch
+          // head-major over all new rows (the query tiles of consecutive problems then adjoin)
           const int g = h / p.grp, hl = h - g * p.grp;
-          const int64_t dst_row = (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
-                                  static_cast<int64_t>(i) * p.grp + hl;
+          const int64_t dst_row =
+              p.problems ? static_cast<int64_t>(g) * p.qrows_g + row * p.grp + hl
+                         : (gm.new_row * p.h_kv + static_cast<int64_t>(g) * gm.n_new) * p.grp +
+                               static_cast<int64_t>(i) * p.grp + hl;
           dst = qhat + dst_row * D;
         } else {
           dst = khat + (row * p.h_kv + (h - p.h_q)) * D;
@@ -158,25 +226,75 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
 // Attention forward
 // ---------------------------------------------------------------------------
 
-// One work unit: a pair of query tiles of one (problem, kv head).
+// One work unit: a pair of query tiles of one kv head, either of one problem or, with
+// packed units, of the packed rows of consecutive problems (gm then describes the
+// unit's key stream: the shared cache prefix [0, c_max) and the new rows [nr_lo, nr_hi)).
 struct Unit {
   Geom gm;
-  int prob, g, qt0, rows_q, n_csub, n_nsub, nt;
-  bool two, valid;
+  int prob, g, qt0, n_csub, n_nsub, nt;
+  int urows;      // query rows (query x head-in-group) of the unit from its first tile on
+  int64_t orow0;  // packed row of the unit's first query: query = packed / grp, head-in-group = packed % grp
+  int64_t qrow0;  // ragged batches: its row in the kv head's block of the rotated queries
+  bool two, valid, packed;
 };
 
-__device__ __forceinline__ Unit make_unit(const AttnParams& p, int u) {
+// The kernel-wide unit plan: packed units from the device plan, else problem units.
+struct UnitPlan {
+  bool packed;
+  int n_pairs, total_units;
+  int64_t cache_row;
+};
+
+__device__ __forceinline__ UnitPlan read_plan(const AttnParams& p) {
+  UnitPlan up{false, 0, p.total_units, 0};
+  if (p.plan) {
+    const AttnPlanHdr h = *p.plan;
+    if (h.packed) {
+      up.packed = true;
+      up.n_pairs = h.n_pairs;
+      up.total_units = h.n_pairs * p.h_kv;
+      up.cache_row = h.cache_row;
+    }
+  }
+  return up;
+}
+
+__device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& up, int u) {
   Unit w;
-  const int pg = u / p.units_per_pg;
-  const int pair = u - pg * p.units_per_pg;
-  w.prob = pg / p.h_kv;
-  w.g = pg - w.prob * p.h_kv;
-  w.gm = problem_geom(p, w.prob);
-  w.rows_q = w.gm.n_new * p.grp;
-  const int n_qt = (w.rows_q + kBM - 1) / kBM;
-  w.qt0 = 2 * pair;
-  w.valid = w.qt0 < n_qt;
-  w.two = w.qt0 + 1 < n_qt;
+  if (up.packed) {
+    // most keys first: pairs in decreasing order (a later pair's problems have longer prefixes
+    // in a block sweep), the kv heads of one pair on neighbouring CTAs (shared K/V in L2)
+    const int pair_rev = u / p.h_kv;
+    w.g = u - pair_rev * p.h_kv;
+    const AttnPlanUnit pu = reinterpret_cast<const AttnPlanUnit*>(p.plan + 1)[up.n_pairs - 1 - pair_rev];
+    w.prob = -1;
+    w.gm.new_row = pu.nr_lo;
+    w.gm.cache_row = up.cache_row;
+    w.gm.n_new = static_cast<int32_t>(pu.nr_hi - pu.nr_lo);
+    w.gm.n_cache = pu.c_max;
+    w.qt0 = 0;
+    w.urows = pu.rows;
+    w.orow0 = pu.p0;
+    w.qrow0 = pu.p0;
+    w.valid = true;
+    w.two = pu.rows > kBM;
+    w.packed = true;
+  } else {
+    const int pg = u / p.units_per_pg;
+    const int pair = u - pg * p.units_per_pg;
+    w.prob = pg / p.h_kv;
+    w.g = pg - w.prob * p.h_kv;
+    w.gm = problem_geom(p, w.prob);
+    const int rows_q = w.gm.n_new * p.grp;
+    const int n_qt = (rows_q + kBM - 1) / kBM;
+    w.qt0 = 2 * pair;
+    w.urows = rows_q - w.qt0 * kBM;
+    w.orow0 = w.gm.new_row * p.grp + w.qt0 * kBM;
+    w.qrow0 = w.orow0;
+    w.valid = w.qt0 < n_qt;
+    w.two = w.qt0 + 1 < n_qt;
+    w.packed = false;
+  }
   w.n_csub = (w.gm.n_cache + kSub - 1) / kSub;
   w.n_nsub = (w.gm.n_new + kSub - 1) / kSub;
   w.nt = (w.n_csub + w.n_nsub + 3) / 4;
@@ -203,6 +321,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool uniform = p.problems == nullptr;
+  const UnitPlan up = read_plan(p);
 
   // No control flow in this kernel depends on the lane: each warp walks its loop
   // as one converged path and a single lane issues through predicated
@@ -255,8 +374,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int qcount = 0;  // units whose Q was loaded
       int fills = 0;   // tiles loaded into this ring so far (all units)
       const int nst = half ? kVStages : kKStages;
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit w = make_unit(p, u);
+      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         if (!half) {
           if (qcount > 0) ok = warp_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
@@ -269,8 +388,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
               qy = (w.qt0 + x) * kBM;
               qz = w.prob * p.h_kv + w.g;
             } else {
-              qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp) +
-                   (w.qt0 + x) * kBM;
+              qy = static_cast<int>(static_cast<int64_t>(w.g) * p.qrows_g + w.qrow0) + x * kBM;
               qz = 0;
             }
 #pragma unroll
@@ -340,8 +458,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int ucount = 0;            // units processed
       int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
       int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit w = make_unit(p, u);
+      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         ok = warp_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
         if (!ok) break;
@@ -447,8 +565,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         ++d;
         return true;
       };
-      for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-        const Unit w = make_unit(p, u);
+      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+        const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
         const int n_jobs = w.two ? 2 * w.nt : w.nt;
@@ -477,26 +595,51 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     bool ok = true;
     int sj = 0;       // S tiles consumed by this slot (all units)
     int merges = 0;   // split-key merges done
-    for (int u = blockIdx.x; u < p.total_units && ok; u += gridDim.x) {
-      const Unit w = make_unit(p, u);
+    for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+      const Unit w = make_unit(p, up, u);
       if (!w.valid) continue;
       const int jobs = w.two ? w.nt : (x == 0 ? (w.nt + 1) / 2 : w.nt / 2);
       float m_run = -INFINITY, l_run = 0.f;
+      // this thread's query row within the unit; with packed units, its own problem's keys:
+      // cache rows below lim, new rows [nlo, nhi) (rows past the unit's end see every key;
+      // their outputs are not stored).  Loads are clamped in range rather than branched around.
+      const int pr_u = (w.two ? x : 0) * kBM + row;
+      int lim = w.gm.n_cache;
+      int64_t nlo = w.gm.new_row, nhi = w.gm.new_row + w.gm.n_new;
+      if (w.packed) {
+        const bool mine = pr_u < w.urows;
+        const int b = p.row_prob[(w.orow0 + min(pr_u, w.urows - 1)) / p.grp];
+        const ssm_attn_problem q = p.problems[b];
+        lim = mine ? q.n_cache : lim;
+        nlo = mine ? q.new_row : nlo;
+        nhi = mine ? q.new_row + q.n_new : nhi;
+      }
       for (int k = 0; k < jobs; ++k) {
         const int j = w.two ? k : 2 * k + x;
         ok = warp_wait(&bars[S_FULL + x], sj & 1, p.wait_ns);
         if (!ok) break;
         tc_fence_after_sync();
         uint32_t sr[kBN];
-        int vcnt[4];
-        const bool full_tile = tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, vcnt);
-        // this row's scores of the tile, keys past a segment end at -inf
+        // valid keys of each 32-key sub-box of the tile for this row: columns [lo, hi)
+        int lo[4], hi[4];
+        bool full_row;
+        if (w.packed) {
+          full_row = row_sub_bounds(j, w.n_csub, w.n_nsub, w.gm.new_row, lim, nlo, nhi, lo, hi);
+        } else {
+          full_row = tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, hi);
+#pragma unroll
+          for (int s4 = 0; s4 < 4; ++s4) lo[s4] = 0;
+        }
+        const bool full_tile = __all_sync(0xffffffffu, full_row);
+        // this row's scores of the tile, invalid keys at -inf (selects, no branch per row)
         auto load_s = [&]() {
           tmem_ld_x128(tS, sr);
           if (!full_tile) {
 #pragma unroll
-            for (int c = 0; c < kBN; ++c)
-              if ((c & (kSub - 1)) >= vcnt[c / kSub]) sr[c] = __float_as_uint(-INFINITY);
+            for (int c = 0; c < kBN; ++c) {
+              const int cc = c & (kSub - 1);
+              sr[c] = (cc >= lo[c / kSub] && cc < hi[c / kSub]) ? sr[c] : __float_as_uint(-INFINITY);
+            }
           }
         };
         load_s();
@@ -529,9 +672,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         };
         float lt;
         if (k == 0) {
-          // the slot's first tile of the unit sets the reference m: its row maximum (finite:
-          // every key tile holds at least one valid key)
-          m_run = row_max() * sc;
+          // the slot's first tile of the unit sets the reference m: its row maximum (0 for a row
+          // with no valid key in this tile, which packed units can give: its first p are then 0)
+          const float mx0 = row_max();
+          m_run = mx0 == -INFINITY ? 0.f : mx0 * sc;
           lt = exp_pass(m_run);
         } else {
           // later tiles: exponentials against the current reference without a row maximum.
@@ -593,10 +737,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         ++merges;
       }
       if (w.two || x == 0) {
-        const int pr = (w.qt0 + (w.two ? x : 0)) * kBM + row;  // packed (query, head-in-group) row
-        const bool valid = pr < w.rows_q;
-        const int qi = pr / p.grp;
-        const int h = w.g * p.grp + (pr - qi * p.grp);
+        const bool valid = pr_u < w.urows;
+        const int64_t prow = w.orow0 + pr_u;    // packed (query, head-in-group) row
+        const int64_t qrow = prow / p.grp;      // the query's new row
+        const int h = w.g * p.grp + static_cast<int>(prow - qrow * p.grp);
         const float m = fmaxf(m_run, mB);
         const float ea = ex2_approx(m_run - m), eb = ex2_approx(mB - m);
         const float a = (l_run > 0.f) ? ea : 0.f;
@@ -604,7 +748,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const float lsum = a * l_run + b * lB;
         const float inv = 1.f / lsum;
         const float ca = a * inv, cb = b * inv;
-        __nv_bfloat16* dst = p.out + ((w.gm.new_row + qi) * p.h_q + h) * D;
+        __nv_bfloat16* dst = p.out + (qrow * p.h_q + h) * D;
 #pragma unroll
         for (int ch = 0; ch < D / 32; ++ch) {
           uint32_t o[32];
@@ -625,7 +769,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
                                          pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7])),
                               valid);
         }
-        if (p.lse) st_global_f32_pred(p.lse + (w.gm.new_row + qi) * p.h_q + h, (m + log2f(lsum)) * kLn2, valid);
+        if (p.lse) st_global_f32_pred(p.lse + qrow * p.h_q + h, (m + log2f(lsum)) * kLn2, valid);
         // this slot's O (and, with split keys, slot B's O too) may now be overwritten
         tc_fence_before_sync();
         warp_arrive(&bars[O_FREE + x]);
@@ -682,6 +826,25 @@ bool make_map(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, 
 // The two launches of an attention call: the rotary/packing pre-pass and the forward.
 constexpr int kPartBoth = 0, kPartRotate = 1, kPartCore = 2;
 
+// Workspace of an attention call (byte offsets, each region 256-byte aligned): rotated
+// queries, rotated new keys, the unit plan of a ragged batch (header, then up to
+// max_pairs packed units) and the problem index of every new row.
+struct WsLayout {
+  size_t khat, plan, row_prob, total;
+  int max_pairs;
+};
+
+WsLayout ws_layout(int64_t total_new, int32_t h_q, int32_t h_kv, int32_t d) {
+  WsLayout l;
+  const int64_t grp = h_q / std::max(h_kv, 1);
+  l.max_pairs = static_cast<int>((total_new * grp + 2 * kBM - 1) / (2 * kBM));
+  l.khat = align_up(static_cast<size_t>(total_new) * h_q * d * 2, 256);
+  l.plan = l.khat + align_up(static_cast<size_t>(total_new) * h_kv * d * 2, 256);
+  l.row_prob = l.plan + align_up(sizeof(AttnPlanHdr) + static_cast<size_t>(l.max_pairs) * sizeof(AttnPlanUnit), 256);
+  l.total = l.row_prob + align_up(static_cast<size_t>(total_new) * sizeof(int32_t), 256);
+  return l;
+}
+
 std::atomic<int> g_attention_variant{SSM_ATTN_AUTO};
 
 int attention_variant() { return g_attention_variant.load(); }
@@ -697,9 +860,9 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   const int grp = h_q / h_kv;
   const int64_t nb = uniform ? batch_or_np : 1;
   const int64_t total_new = uniform ? static_cast<int64_t>(batch_or_np) * new_rows_per_b : new_rows_per_b;
+  const WsLayout wl = ws_layout(total_new, h_q, h_kv, D);
   auto* qhat = static_cast<__nv_bfloat16*>(workspace);
-  auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) +
-                                                align_up(static_cast<size_t>(total_new) * h_q * D * 2, 256));
+  auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) + wl.khat);
   // which kernel: 128-row query tiles unless key tiles (queries on the MMA N dimension)
   // are requested and every (problem, kv head) has at most kKtMaxRows query rows
   const bool kt_fits = D == 128 && static_cast<int64_t>(max_n_new) * grp <= kKtMaxRows;
@@ -745,6 +908,9 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.h_kv = h_kv;
   p.grp = grp;
   p.new_rows_extent = static_cast<int32_t>(new_rows_per_b);
+  p.qrows_g = uniform ? 0 : static_cast<int32_t>(total_new * grp);
+  p.plan = uniform ? nullptr : reinterpret_cast<AttnPlanHdr*>(static_cast<uint8_t*>(workspace) + wl.plan);
+  p.row_prob = uniform ? nullptr : reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob);
   p.scale_log2 = scale * kLog2e;
   p.out = static_cast<__nv_bfloat16*>(out);
   p.lse = lse;
@@ -757,7 +923,8 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, 3ll * num_sms()));
     rope_pack_kernel<D><<<grid, kRopeWarps * 32, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
                                                           static_cast<const __nv_bfloat16*>(k_new), pos, p,
-                                                          rope_theta, max_n_new, n_prob, qhat, khat);
+                                                          rope_theta, max_n_new, n_prob, wl.max_pairs, qhat,
+                                                          khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK || part == kPartRotate) return s;
   }
@@ -796,7 +963,9 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   const int64_t total_units = static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
   if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
   p.total_units = static_cast<int32_t>(total_units);
-  const int grid = static_cast<int>(std::min<int64_t>(total_units, num_sms()));
+  // a ragged batch may run packed units instead (decided on the device by the pre-pass)
+  const int64_t max_units = uniform ? total_units : std::max<int64_t>(total_units, int64_t{wl.max_pairs} * h_kv);
+  const int grid = static_cast<int>(std::min<int64_t>(max_units, num_sms()));
   attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128, m.kn128,
                                                            m.vn128, p);
   return launch_status();
@@ -829,8 +998,7 @@ ssm_status ssm_set_attention_variant(int32_t variant) {
 
 size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv, int32_t head_dim) {
   if (total_new_rows <= 0 || h_q <= 0 || h_kv <= 0 || head_dim <= 0) return 0;
-  return ssm::align_up(static_cast<size_t>(total_new_rows) * h_q * head_dim * 2, 256) +
-         ssm::align_up(static_cast<size_t>(total_new_rows) * h_kv * head_dim * 2, 256);
+  return ssm::ws_layout(total_new_rows, h_q, h_kv, head_dim).total;
 }
 
 ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,

@@ -33,11 +33,33 @@ constexpr float kSpecSumMax = 65536.0f;  // a tile's row sum of p above this tak
 constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kDrainNs = 200000000ull;
 
+// Packed units (ragged batches whose problems share one cache prefix and whose new rows
+// follow one another): the rows of consecutive problems fill the query tiles together
+// instead of each problem padding its own last tile.  A unit is a pair of 128-row tiles
+// of one kv head's packed rows; its keys are the cache rows [0, c_max) followed by the
+// new rows [nr_lo, nr_hi) of the problems it touches, and each row sees only its own
+// problem's cache prefix and new rows.  The plan is made on the device by the RoPE
+// pre-pass and read by the forward kernel.
+struct AttnPlanHdr {
+  int32_t packed;     // 1: the units below; 0: one problem per unit
+  int32_t n_pairs;    // packed units per kv head
+  int64_t cache_row;  // the shared cache's first row
+  int64_t pad[2];
+};
+struct AttnPlanUnit {
+  int32_t p0, rows;   // first packed row (query x head-in-group, within the kv head's block), rows (<= 256)
+  int32_t c_max, pad; // cache keys: the largest prefix among the unit's problems
+  int64_t nr_lo, nr_hi;  // new keys: the unit's problems' new rows
+};
+
 struct AttnParams {
   const ssm_attn_problem* problems;  // null: uniform batch
   int32_t n_new_u, n_cache_u;
   int32_t h_q, h_kv, grp;
   int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
+  int32_t qrows_g;                   // ragged batches: rotated query rows of one kv head (head-major layout)
+  AttnPlanHdr* plan;                 // ragged batches: the unit plan (header, then units), else null
+  int32_t* row_prob;                 // ragged batches: problem of each new row
   int32_t units_per_pg;              // work units per (problem, kv head)
   int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)
@@ -72,6 +94,31 @@ __device__ __forceinline__ Geom problem_geom(const AttnParams& p, int prob) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// This row's valid key range in each 32-row sub-box of key tile j of a packed unit: cache keys
+// below the row's own prefix `lim`; new keys within the row's own problem [nlo, nhi).  The
+// valid keys of a sub-box are columns [lo, hi); returns true if all 128 are valid.
+__device__ __forceinline__ bool row_sub_bounds(int j, int n_csub, int n_nsub, int64_t nr_lo, int lim, int64_t nlo,
+                                               int64_t nhi, int (&lo)[4], int (&hi)[4]) {
+  bool full = true;
+#pragma unroll
+  for (int s4 = 0; s4 < 4; ++s4) {
+    const int sub = 4 * j + s4;
+    int a = 0, b = 0;
+    if (sub < n_csub) {
+      b = max(0, min(kSub, lim - sub * kSub));
+    } else if (sub - n_csub < n_nsub) {
+      const int64_t kn = nr_lo + static_cast<int64_t>(sub - n_csub) * kSub;
+      const int64_t da = nlo - kn, db = nhi - kn;  // clamped to [0, kSub]
+      a = da < 0 ? 0 : (da > kSub ? kSub : static_cast<int>(da));
+      b = db < 0 ? 0 : (db > kSub ? kSub : static_cast<int>(db));
+    }
+    lo[s4] = a;
+    hi[s4] = max(a, b);
+    full = full && a == 0 && b == kSub;
+  }
+  return full;
 }
 
 // Valid keys in each 32-row sub-box of key tile j (cache sub-boxes first, then

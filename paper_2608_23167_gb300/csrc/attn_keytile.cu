@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
             qy = 0;
             qz = w.prob * p.h_kv + w.g;
           } else {
-            qy = static_cast<int>((w.gm.new_row * p.h_kv + static_cast<int64_t>(w.g) * w.gm.n_new) * p.grp);
+            qy = static_cast<int>(static_cast<int64_t>(w.g) * p.qrows_g + w.gm.new_row * p.grp);
             qz = 0;
           }
           if (w.qs) {

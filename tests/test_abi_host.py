@@ -90,7 +90,15 @@ def test_argument_validation_without_device(lib):
 def test_workspace_sizes(lib):
     from paper_2608_23167_gb300 import ssm
     import torch
-    assert ssm.ssm_attention_workspace_size(101 * 8, 32, 32, 128) == 2 * 101 * 8 * 32 * 128 * 2
+    # rotated queries and keys, then the unit plan (32-byte header, 32 bytes per packed unit of
+    # 256 query rows of a kv head) and the problem index of every new row, each region 256-aligned
+    up = lambda x: (x + 255) // 256 * 256
+    rows, pairs = 101 * 8, (101 * 8 + 255) // 256
+    assert ssm.ssm_attention_workspace_size(rows, 32, 32, 128) == (
+        2 * rows * 32 * 128 * 2 + up(32 + 32 * pairs) + up(4 * rows))
+    rows, pairs = 8854, (8854 * 7 + 255) // 256    # GQA: 7 query heads per kv head pack 7 rows per query
+    assert ssm.ssm_attention_workspace_size(rows, 28, 4, 128) == (
+        up(rows * 28 * 256) + up(rows * 4 * 256) + up(32 + 32 * pairs) + up(4 * rows))
     # 126464 bf16 entries are 16 stages of 8192; segments aim at 2048 work items per call
     ws = ssm.ssm_unmask_workspace_size(8, 32, 126464, torch.bfloat16)
     assert ws == 8 * 32 * 8 * 16   # 256 rows: eight segments of two stages each, 16-byte partials

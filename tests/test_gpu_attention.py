@@ -310,3 +310,56 @@ def test_attention_varlen_cold_l2_and_graph_replay(dev, variant, shape):
         assert torch.equal(out, ref)
     finally:
         ssm.ssm_set_wait_limit_ns(0)
+
+
+@pytest.mark.parametrize("case", ["mixed", "gqa", "d64", "one_row"])
+def test_attention_varlen_packed_prefix(dev, variant, case):
+    """Ragged batches whose problems read prefixes of one shared cache and whose new rows
+    follow one another: the kernel packs the rows of consecutive problems into shared query
+    tiles (each row masked to its own prefix and its own new rows).  Every problem is checked
+    against the oracle: problems without cache rows next to ones with long prefixes, problems
+    straddling a tile pair, GQA packing (several query heads per kv head), d = 64, and one-row
+    problems (hundreds per tile pair); the last pair has at most 128 rows (split keys)."""
+    from paper_2608_23167_gb300 import ssm
+    h_q, h_kv, d, theta = 4, 4, 128, 1e4
+    if case == "mixed":
+        sizes = [(37, 100), (1, 0), (130, 250), (64, 250), (5, 31), (200, 512), (33, 64)]
+    elif case == "gqa":
+        h_q, h_kv = 8, 2
+        sizes = [(50, 300), (70, 320), (20, 0), (90, 400)]
+    elif case == "d64":
+        d = 64
+        sizes = [(37, 100), (1, 0), (130, 250), (64, 250), (5, 31), (200, 512), (33, 64)]
+    else:
+        sizes = [(1, (7 * i) % 200) for i in range(300)]
+    if variant == "key_tiles" and not _key_tiles_fit(max(n for n, _ in sizes), h_q, h_kv, d):
+        pytest.skip("shape outside the key-tile kernel")
+    cache_rows = max(c for _, c in sizes) or 1
+    rows, new_row = [], 0
+    for n, c in sizes:
+        rows.append((new_row, 0, n, c))
+        new_row += n
+    seed = 91 + len(sizes) + d
+    q = W.draw_normal_bf16((new_row, h_q, d), 1.0, seed)
+    k = W.draw_normal_bf16((new_row, h_kv, d), 1.0, seed + 1)
+    v = W.draw_normal_bf16((new_row, h_kv, d), 1.0, seed + 2)
+    kc = W.draw_normal_bf16((cache_rows, h_kv, d), 1.0, seed + 3)
+    vc = W.draw_normal_bf16((cache_rows, h_kv, d), 1.0, seed + 4)
+    g = torch.Generator().manual_seed(seed + 5)
+    pos = torch.cat([(c + torch.randperm(2 * n + 3, generator=g)[:n]) for n, c in sizes]).to(torch.int32)
+    out = torch.full((new_row, h_q, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    lse = torch.full((new_row, h_q), float("nan"), dtype=torch.float32, device=dev)
+    ssm.ssm_attention_varlen(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev),
+                             ssm.attn_problems_tensor(rows, dev), len(rows), max(n for n, _ in sizes),
+                             max(c for _, c in sizes), out, theta, lse=lse)
+    torch.cuda.synchronize()
+    check_device_error()
+    og, lg = f64(out), f64(lse)
+    for i, (nr, _, n, c) in enumerate(rows):
+        if case == "one_row" and i % 10:
+            continue
+        sl = slice(nr, nr + n)
+        ref, ref_lse = O.attention(f64(q[None, sl]), f64(k[None, sl]), f64(v[None, sl]), pos[sl].numpy(),
+                                   f64(kc[None, :c]) if c else None, f64(vc[None, :c]) if c else None, theta)
+        assert_attention_close(og[sl][None], ref, f"{case} problem {i} ({n} rows, prefix {c})")
+        assert np.abs(lg[sl][None] - ref_lse).max() <= 2e-2, f"{case} problem {i} lse"
