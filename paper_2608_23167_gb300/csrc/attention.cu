@@ -245,9 +245,12 @@ struct UnitPlan {
   int64_t cache_row;
 };
 
+// PACKABLE = false compiles the kernel without packed units at all (no plan read, no per-row
+// key bounds in the softmax): the host launches that form for batches that cannot pack.
+template <bool PACKABLE>
 __device__ __forceinline__ UnitPlan read_plan(const AttnParams& p) {
   UnitPlan up{false, 0, p.total_units, 0};
-  if (p.plan) {
+  if (PACKABLE && p.plan) {
     const AttnPlanHdr h = *p.plan;
     if (h.packed) {
       up.packed = true;
@@ -301,7 +304,7 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
   return w;
 }
 
-template <int D>
+template <int D, bool PACKABLE>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
     const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kn,
@@ -321,7 +324,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool uniform = p.problems == nullptr;
-  const UnitPlan up = read_plan(p);
+  const UnitPlan up = read_plan<PACKABLE>(p);
 
   // No control flow in this kernel depends on the lane: each warp walks its loop
   // as one converged path and a single lane issues through predicated
@@ -849,11 +852,40 @@ std::atomic<int> g_attention_variant{SSM_ATTN_AUTO};
 
 int attention_variant() { return g_attention_variant.load(); }
 
+// One instantiation of the forward: the register split assumes the compiled register count
+// (checked once), the dynamic shared memory is opted into once per device.
+template <int D, bool PACKABLE>
+ssm_status launch_fwd(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
+  using L = Layout<D>;
+  static std::atomic<int> regs_ok{0};  // 0 unknown, 1 ok, 2 mismatch
+  int st_regs = regs_ok.load();
+  if (st_regs == 0) {
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, PACKABLE>) != cudaSuccess) return SSM_ERR_CUDA;
+    st_regs = fa.numRegs == kLaunchRegs ? 1 : 2;
+    regs_ok.store(st_regs);
+  }
+  if (st_regs != 1) return SSM_ERR_UNSUPPORTED;
+  static std::atomic<uint64_t> attr_set{0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(attr_set.load() & bit)) {
+    if (cudaFuncSetAttribute(attn_fwd_kernel<D, PACKABLE>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
+        cudaSuccess)
+      return SSM_ERR_CUDA;
+    attr_set.fetch_or(bit);
+  }
+  attn_fwd_kernel<D, PACKABLE><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
+                                                                     m.kn128, m.vn128, p);
+  return launch_status();
+}
+
 template <int D>
 ssm_status launch_attention(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
                             const void* k_cache, const void* v_cache, bool uniform, int32_t batch_or_np,
                             int64_t new_rows_per_b, int64_t cache_rows_per_b, int32_t max_n_new,
-                            const ssm_attn_problem* problems, int32_t h_q, int32_t h_kv,
+                            int32_t max_n_cache, const ssm_attn_problem* problems, int32_t h_q, int32_t h_kv,
                             float rope_theta, float scale, void* out, float* lse, void* workspace,
                             cudaStream_t st, int part = kPartBoth) {
   using L = Layout<D>;
@@ -909,8 +941,13 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.grp = grp;
   p.new_rows_extent = static_cast<int32_t>(new_rows_per_b);
   p.qrows_g = uniform ? 0 : static_cast<int32_t>(total_new * grp);
-  p.plan = uniform ? nullptr : reinterpret_cast<AttnPlanHdr*>(static_cast<uint8_t*>(workspace) + wl.plan);
-  p.row_prob = uniform ? nullptr : reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob);
+  // Packed units need every problem to read one shared cache; a cache too small to hold two of
+  // the longest prefixes (or no cache at all) is the only candidate.  Other batches run the
+  // forward compiled without packed units, and the pre-pass makes no plan for them.
+  const bool may_pack = !uniform && !use_kt && batch_or_np >= 2 &&
+                        (cache_rows_per_b == 0 || 2 * static_cast<int64_t>(max_n_cache) > cache_rows_per_b);
+  p.plan = may_pack ? reinterpret_cast<AttnPlanHdr*>(static_cast<uint8_t*>(workspace) + wl.plan) : nullptr;
+  p.row_prob = may_pack ? reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob) : nullptr;
   p.scale_log2 = scale * kLog2e;
   p.out = static_cast<__nv_bfloat16*>(out);
   p.lse = lse;
@@ -935,40 +972,15 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     p.total_units = static_cast<int32_t>(total_units);
     return launch_attn_keytile(m, p, static_cast<int>(std::min<int64_t>(total_units, num_sms())), st);
   }
-  // the warpgroup register split assumes the compiled register count
-  {
-    static std::atomic<int> regs_ok{0};  // 0 unknown, 1 ok, 2 mismatch
-    int st_regs = regs_ok.load();
-    if (st_regs == 0) {
-      cudaFuncAttributes fa;
-      if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D>) != cudaSuccess) return SSM_ERR_CUDA;
-      st_regs = fa.numRegs == kLaunchRegs ? 1 : 2;
-      regs_ok.store(st_regs);
-    }
-    if (st_regs != 1) return SSM_ERR_UNSUPPORTED;
-  }
-  // the dynamic shared-memory opt-in is a per-device function attribute
-  static std::atomic<uint64_t> attr_set{0};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
-  const uint64_t bit = 1ull << (dev & 63);
-  if (!(attr_set.load() & bit)) {
-    if (cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
-        cudaSuccess)
-      return SSM_ERR_CUDA;
-    attr_set.fetch_or(bit);
-  }
   const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
   p.units_per_pg = (m_tiles + 1) / 2;
   const int64_t total_units = static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
   if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
   p.total_units = static_cast<int32_t>(total_units);
-  // a ragged batch may run packed units instead (decided on the device by the pre-pass)
-  const int64_t max_units = uniform ? total_units : std::max<int64_t>(total_units, int64_t{wl.max_pairs} * h_kv);
-  const int grid = static_cast<int>(std::min<int64_t>(max_units, num_sms()));
-  attn_fwd_kernel<D><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128, m.kn128,
-                                                           m.vn128, p);
-  return launch_status();
+  if (!may_pack) return launch_fwd<D, false>(m, p, static_cast<int>(std::min<int64_t>(total_units, num_sms())), st);
+  // packed units, if the pre-pass's plan chose them, number at most max_pairs per kv head
+  const int64_t max_units = std::max<int64_t>(total_units, int64_t{wl.max_pairs} * h_kv);
+  return launch_fwd<D, true>(m, p, static_cast<int>(std::min<int64_t>(max_units, num_sms())), st);
 }
 
 ssm_status check_attn(const void* q, const void* k_new, const void* v_new, const int32_t* pos,
@@ -1019,9 +1031,9 @@ ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, co
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (head_dim == 128)
     return ssm::launch_attention<128>(q, k_new, v_new, pos, k_cache, v_cache, true, batch, n_new, n_cache, n_new,
-                                      nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
+                                      n_cache, nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
   return ssm::launch_attention<64>(q, k_new, v_new, pos, k_cache, v_cache, true, batch, n_new, n_cache, n_new,
-                                   nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
+                                   n_cache, nullptr, h_q, h_kv, rope_theta, scale, out, lse, workspace, st);
 }
 
 static ssm_status attention_varlen_part(int part, const void* q, const void* k_new, const void* v_new,
@@ -1046,11 +1058,11 @@ static ssm_status attention_varlen_part(int part, const void* q, const void* k_n
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (head_dim == 128)
     return ssm::launch_attention<128>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
-                                      total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out,
-                                      lse, workspace, st, part);
+                                      total_cache_rows, max_n_new, max_n_cache, problems, h_q, h_kv, rope_theta,
+                                      scale, out, lse, workspace, st, part);
   return ssm::launch_attention<64>(q, k_new, v_new, pos, k_cache, v_cache, false, n_problems, total_new_rows,
-                                   total_cache_rows, max_n_new, problems, h_q, h_kv, rope_theta, scale, out, lse,
-                                   workspace, st, part);
+                                   total_cache_rows, max_n_new, max_n_cache, problems, h_q, h_kv, rope_theta, scale,
+                                   out, lse, workspace, st, part);
 }
 
 
