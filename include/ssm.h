@@ -199,7 +199,8 @@ ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t
  *   lse          fp32 [batch, n_new, h_q]  natural-log sum-exp of the scaled
  *                scores (may be NULL)
  *   workspace    >= ssm_attention_workspace_size(batch * n_new, h_q, h_kv, d)
- *                bytes, 256-byte aligned; holds the rotated queries and keys.
+ *                bytes, 256-byte aligned; holds the rotated queries and keys
+ *                (and, for the ragged form, the work plan and a row map).
  * d in {64, 128}; h_q % h_kv == 0; every pointer 16-byte aligned. */
 size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv,
                                     int32_t head_dim);
@@ -217,7 +218,12 @@ ssm_status ssm_attention(const void* q, const void* k_new, const void* v_new, co
  * [total_cache_rows, h_kv, d]; several problems may share cache rows).
  * max_n_new / max_n_cache bound the per-problem sizes (grid size).  A tile at
  * the ragged end of a problem may read rows of the same buffers beyond it
- * (multiplied by an exact zero): keep every row of the packed buffers finite. */
+ * (multiplied by an exact zero): keep every row of the packed buffers finite.
+ * When every problem reads one shared cache (equal cache_row; prefixes of
+ * different lengths, e.g. the block indices of one sequence) and the problems'
+ * new rows follow one another from row 0, the rows of consecutive problems may
+ * share query tiles (each row still sees only its own prefix and its own new
+ * rows); the result is the same either way. */
 typedef struct {
   int64_t new_row;
   int64_t cache_row;
@@ -236,9 +242,10 @@ ssm_status ssm_attention_varlen(const void* q, const void* k_new, const void* v_
 
 /* The two launches ssm_attention_varlen makes, as separate calls with the same
  * arguments, for a caller that schedules or times them apart:
- *   ..._rotate writes the rotated queries (packed by GQA group) and the rotated
- *              new keys into `workspace` (the RoPE pre-pass; q, k_new, pos and
- *              the problem table are read, v/cache/out/lse are not touched);
+ *   ..._rotate writes the rotated queries (packed by GQA group), the rotated
+ *              new keys and the work plan into `workspace` (the RoPE pre-pass;
+ *              q, k_new, pos and the problem table are read, v/cache/out/lse
+ *              are not touched);
  *   ..._core   runs the attention forward from that workspace (q, k_new and pos
  *              are not read again).
  * ..._core must follow a ..._rotate with the same arguments and workspace, in
