@@ -3,8 +3,8 @@
 //
 // Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
 // segments of whole 16 KB chunks (the work items, dealt round-robin to
-// persistent CTAs, six per SM): one segment per row once a call has 2048 rows,
-// shorter ones for smaller calls.  Each thread streams its own 64-byte slices of successive
+// persistent CTAs, three per SM, one wave): one segment per row once a call has
+// 912 rows, shorter ones for smaller calls (about two items per CTA).  Each thread streams its own 64-byte slices of successive
 // 16 KB chunks from HBM into a private two-stage shared-memory ring with
 // 16-byte cp.async copies, so the read runs ahead of the arithmetic without any
 // barrier (a thread only reads back what it copied itself), and folds every
@@ -30,7 +30,7 @@ namespace ssm {
 namespace {
 
 constexpr int kUnmaskThreads = 256;
-constexpr int64_t kItemsTarget = 2048;             // segments (work items) a call aims for
+constexpr int64_t kItemsTarget = 912;              // segments (work items) a call aims for: ~2 per resident CTA
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Partial {
@@ -327,8 +327,18 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
     const int64_t row = b * block_len + j;
     mj = masked[row] != 0;
     if (mj) {
-      Partial p = part[row * n_chunks];
-      for (int c = 1; c < n_chunks; ++c) p = merge(p, part[row * n_chunks + c]);
+      // the row's partials are loaded eight at a time, independently, then merged (a chain
+      // of dependent loads would cost one memory latency per partial)
+      const Partial* pr = part + row * n_chunks;
+      Partial p = pr[0];
+      for (int c0 = 1; c0 < n_chunks; c0 += 8) {
+        Partial q[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) q[c] = pr[min(c0 + c, n_chunks - 1)];
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          if (c0 + c < n_chunks) p = merge(p, q[c]);
+      }
       const float inv = 1.f / p.s;                     // largest probability = 1 / sum exp(x - max)
       cj = inv;
       p2 = (p.m2 > -INFINITY) ? ex2((p.m2 - p.m) * kLog2e) * inv : 0.f;
@@ -445,7 +455,8 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));
   const size_t stream_smem = ssm::kStreamStages * ssm::kStageBytes + 128;  // 96 KB: two CTAs per SM
   const int64_t n_items = rows * plan.n_chunks;
-  const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 6 * ssm::num_sms()));
+  // one wave: three CTAs per SM are resident (registers), each takes ~2 items of ~kItemsTarget
+  const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 3 * ssm::num_sms()));
   unsigned* err = ssm::device_error_word();
   const uint64_t wait_ns = ssm::wait_limit_ns();
   const bool need_second = p2 != nullptr || mode == SSM_COMMIT_MARGIN;
