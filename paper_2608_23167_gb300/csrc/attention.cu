@@ -238,6 +238,17 @@ struct Unit {
   bool two, valid, packed;
 };
 
+// Units are dealt to the persistent CTAs in waves of gridDim.x, each wave in the opposite
+// direction to the last ("snake" order): with units sorted by decreasing cost, a CTA that took
+// a heavy unit in one wave takes a light one in the next, which evens out the CTAs' totals
+// (on the long sweep the simulated makespan falls from 9 % to 6 % above the mean).  Every
+// role of a CTA walks the same sequence; it is increasing, so the first unit past the end
+// ends the walk.
+__device__ __forceinline__ int snake_unit(int k) {
+  const int c = static_cast<int>(blockIdx.x), g = static_cast<int>(gridDim.x);
+  return k * g + ((k & 1) ? g - 1 - c : c);
+}
+
 // The kernel-wide unit plan: packed units from the device plan, else problem units.
 struct UnitPlan {
   bool packed;
@@ -377,7 +388,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int qcount = 0;  // units whose Q was loaded
       int fills = 0;   // tiles loaded into this ring so far (all units)
       const int nst = half ? kVStages : kKStages;
-      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+      for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
         const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         if (!half) {
@@ -461,7 +472,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int ucount = 0;            // units processed
       int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
       int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
-      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+      for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
         const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         ok = warp_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
@@ -568,7 +579,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         ++d;
         return true;
       };
-      for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+      for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
         const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
@@ -598,7 +609,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     bool ok = true;
     int sj = 0;       // S tiles consumed by this slot (all units)
     int merges = 0;   // split-key merges done
-    for (int u = blockIdx.x; u < up.total_units && ok; u += gridDim.x) {
+    for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
       const Unit w = make_unit(p, up, u);
       if (!w.valid) continue;
       const int jobs = w.two ? w.nt : (x == 0 ? (w.nt + 1) / 2 : w.nt / 2);
