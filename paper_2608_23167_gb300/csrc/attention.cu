@@ -9,9 +9,12 @@
 //    (query i, head-in-group hl) -> row i * grp + hl, so that a 128-row M tile
 //    of the tensor-core GEMM holds every query head that shares a K/V head.
 //  * attn_fwd_kernel: persistent, one CTA per SM.  Work units are (problem,
-//    kv head, pair of 128-row query tiles), taken round-robin; barrier phases
-//    carry over from unit to unit, so the next unit's Q/K loads and first
-//    QK^T overlap the current unit's last softmax and epilogue.  Per unit,
+//    kv head, pair of 128-row query tiles) or, for ragged batches whose
+//    problems share one cache prefix, pairs of tiles of consecutive problems'
+//    packed rows (each row masked to its own prefix and new rows); they are
+//    dealt in snake order, and barrier phases carry over from unit to unit,
+//    so the next unit's Q/K loads and first QK^T overlap the current unit's
+//    last softmax and epilogue.  Per unit,
 //    warps 0 and 2 stream the K and the V tiles with TMA, each ring at its own
 //    pace (128 keys = four 32-row sub-boxes, so the cache segment and the
 //    new-row segment pack back to back with at most 31 padded keys each;
@@ -22,8 +25,10 @@
 //    while one turns its S tile into P (written back over S as bf16), the
 //    tensor core runs the other slot's GEMMs.  With two query tiles each slot
 //    owns one; with a single query tile the slots split the key tiles
-//    (even/odd) and merge their partial softmax states at the end.  O is
-//    rescaled only when a row maximum grows by more than 2^8.
+//    (even/odd) and merge their partial softmax states at the end.  After a
+//    slot's first tile of a unit the exponentials are taken against the
+//    current reference without a row maximum; O is rescaled only when a
+//    tile's row sum of p exceeds 2^16.
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 

@@ -131,7 +131,7 @@ struct RunState {
 template <typename T, bool NEED_SECOND>
 __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_stream_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
-    const uint8_t* __restrict__ masked, Partial* __restrict__ part, unsigned* err, uint64_t wait_ns) {
+    const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
   constexpr int ESZ = sizeof(T);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
@@ -457,8 +457,6 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   const int64_t n_items = rows * plan.n_chunks;
   // one wave: three CTAs per SM are resident (registers), each takes ~2 items of ~kItemsTarget
   const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 3 * ssm::num_sms()));
-  unsigned* err = ssm::device_error_word();
-  const uint64_t wait_ns = ssm::wait_limit_ns();
   const bool need_second = p2 != nullptr || mode == SSM_COMMIT_MARGIN;
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
@@ -468,10 +466,10 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
         return SSM_ERR_CUDA;
       if (need_second)
         ssm::unmask_stream_kernel<__nv_bfloat16, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::unmask_stream_kernel<__nv_bfloat16, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
     } else {
       ssm::unmask_partial_scalar_kernel<__nv_bfloat16><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
@@ -484,10 +482,10 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
         return SSM_ERR_CUDA;
       if (need_second)
         ssm::unmask_stream_kernel<float, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::unmask_stream_kernel<float, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part, err, wait_ns);
+            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
     } else {
       ssm::unmask_partial_scalar_kernel<float><<<grid, ssm::kUnmaskThreads, 0, st>>>(
           x, vocab, plan.chunk, plan.n_chunks, masked, part);
