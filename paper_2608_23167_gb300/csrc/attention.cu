@@ -623,15 +623,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       // cache rows below lim, new rows [nlo, nhi) (rows past the unit's end see every key;
       // their outputs are not stored).  Loads are clamped in range rather than branched around.
       const int pr_u = (w.two ? x : 0) * kBM + row;
-      int lim = w.gm.n_cache;
-      int64_t nlo = w.gm.new_row, nhi = w.gm.new_row + w.gm.n_new;
+      // (new rows counted from the unit's first new row, which fits 32 bits)
+      int lim = w.gm.n_cache, nlo = 0, nhi = w.gm.n_new;
       if (w.packed) {
         const bool mine = pr_u < w.urows;
         const int b = p.row_prob[(w.orow0 + min(pr_u, w.urows - 1)) / p.grp];
         const ssm_attn_problem q = p.problems[b];
         lim = mine ? q.n_cache : lim;
-        nlo = mine ? q.new_row : nlo;
-        nhi = mine ? q.new_row + q.n_new : nhi;
+        nlo = mine ? static_cast<int>(q.new_row - w.gm.new_row) : nlo;
+        nhi = mine ? static_cast<int>(q.new_row - w.gm.new_row) + q.n_new : nhi;
       }
       for (int k = 0; k < jobs; ++k) {
         const int j = w.two ? k : 2 * k + x;
@@ -643,7 +643,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         int lo[4], hi[4];
         bool full_row;
         if (w.packed) {
-          full_row = row_sub_bounds(j, w.n_csub, w.n_nsub, w.gm.new_row, lim, nlo, nhi, lo, hi);
+          full_row = row_sub_bounds(j, w.n_csub, w.n_nsub, lim, nlo, nhi, lo, hi);
         } else {
           full_row = tile_valid_counts(j, w.n_csub, w.n_nsub, w.gm, hi);
 #pragma unroll
@@ -768,25 +768,44 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const float inv = 1.f / lsum;
         const float ca = a * inv, cb = b * inv;
         __nv_bfloat16* dst = p.out + (qrow * p.h_q + h) * D;
-#pragma unroll
-        for (int ch = 0; ch < D / 32; ++ch) {
-          uint32_t o[32];
-          tmem_ld_x32(tO + ch * 32, o);
-          float f[32];
-#pragma unroll
-          for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[c]) * ca;
-          if (!w.two && w.nt >= 2) {  // warp-uniform; cb = 0 for a row slot B gave no weight
-            tmem_ld_x32(tOB + ch * 32, o);
-#pragma unroll
-            for (int c = 0; c < 32; ++c) f[c] = fmaf(__uint_as_float(o[c]), cb, f[c]);
-          }
-          uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
+        // 32 output columns of this row from fp32 values: bf16, four 16-byte stores
+        auto store32 = [&](int c0, const float (&f)[32]) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c0);
 #pragma unroll
           for (int v = 0; v < 4; ++v)
             st_global_v4_pred(d4 + v,
                               make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
                                          pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7])),
                               valid);
+        };
+        if (!w.two && w.nt >= 2) {
+          // split keys: both accumulators, 64 columns at a time, each pair of loads one round trip
+          // (warp-uniform; cb = 0 for a row slot B gave no weight)
+#pragma unroll
+          for (int hh = 0; hh < D / 64; ++hh) {
+            uint32_t oa[64], ob[64];
+            tmem_ld_x64_pair(tO + hh * 64, tOB + hh * 64, oa, ob);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              float f[32];
+#pragma unroll
+              for (int c = 0; c < 32; ++c)
+                f[c] = fmaf(__uint_as_float(ob[32 * q + c]), cb, __uint_as_float(oa[32 * q + c]) * ca);
+              store32(hh * 64 + q * 32, f);
+            }
+          }
+        } else {
+          // the whole accumulator row in one round trip
+          uint32_t o[D];
+          if constexpr (D == 128) tmem_ld_x128(tO, o);
+          else tmem_ld_x64(tO, o);
+#pragma unroll
+          for (int ch = 0; ch < D / 32; ++ch) {
+            float f[32];
+#pragma unroll
+            for (int c = 0; c < 32; ++c) f[c] = __uint_as_float(o[ch * 32 + c]) * ca;
+            store32(ch * 32, f);
+          }
         }
         if (p.lse) st_global_f32_pred(p.lse + qrow * p.h_q + h, (m + log2f(lsum)) * kLn2, valid);
         // this slot's O (and, with split keys, slot B's O too) may now be overwritten

@@ -97,25 +97,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 }
 
 // This row's valid key range in each 32-row sub-box of key tile j of a packed unit: cache keys
-// below the row's own prefix `lim`; new keys within the row's own problem [nlo, nhi).  The
-// valid keys of a sub-box are columns [lo, hi); returns true if all 128 are valid.
-__device__ __forceinline__ bool row_sub_bounds(int j, int n_csub, int n_nsub, int64_t nr_lo, int lim, int64_t nlo,
-                                               int64_t nhi, int (&lo)[4], int (&hi)[4]) {
+// below the row's own prefix `lim`; new keys within the row's own problem, [nlo, nhi) counted from
+// the unit's first new row.  The valid keys of a sub-box are columns [lo, hi); returns true if all
+// 128 are valid.
+__device__ __forceinline__ bool row_sub_bounds(int j, int n_csub, int n_nsub, int lim, int nlo, int nhi,
+                                               int (&lo)[4], int (&hi)[4]) {
   bool full = true;
 #pragma unroll
   for (int s4 = 0; s4 < 4; ++s4) {
     const int sub = 4 * j + s4;
     int a = 0, b = 0;
     if (sub < n_csub) {
-      b = max(0, min(kSub, lim - sub * kSub));
+      b = lim - sub * kSub;
     } else if (sub - n_csub < n_nsub) {
-      const int64_t kn = nr_lo + static_cast<int64_t>(sub - n_csub) * kSub;
-      const int64_t da = nlo - kn, db = nhi - kn;  // clamped to [0, kSub]
-      a = da < 0 ? 0 : (da > kSub ? kSub : static_cast<int>(da));
-      b = db < 0 ? 0 : (db > kSub ? kSub : static_cast<int>(db));
+      const int kn = (sub - n_csub) * kSub;
+      a = nlo - kn;
+      b = nhi - kn;
     }
+    a = min(max(a, 0), kSub);
+    b = min(max(b, a), kSub);
     lo[s4] = a;
-    hi[s4] = max(a, b);
+    hi[s4] = b;
     full = full && a == 0 && b == kSub;
   }
   return full;
