@@ -104,3 +104,23 @@ def test_workspace_sizes(lib):
     assert ws == 8 * 32 * 4 * 16   # 256 rows: four segments of four stages each, 16-byte partials
     assert ssm.ssm_unmask_workspace_size(64, 32, 126464, torch.bfloat16) == 64 * 32 * 16   # one segment per row
     assert ssm.ssm_unmask_workspace_size(1, 4, 126464, torch.bfloat16) == 4 * 16 * 16      # one stage per segment
+
+
+def test_attention_digest_covers_its_includes():
+    """The bench trusts a recorded DRAM-traffic figure only while its source digest matches the
+    attention forward's sources; every local header attention.cu includes (transitively) must be
+    part of that digest, or a change to it would leave a stale figure in use."""
+    import os
+    import re
+    from paper_2608_23167_gb300 import build_lib
+    seen, todo = set(), ["attention.cu"]
+    while todo:
+        name = todo.pop()
+        if name in seen:
+            continue
+        seen.add(name)
+        with open(os.path.join(build_lib.CSRC, name)) as f:
+            for inc in re.findall(r'^#include "([^"]+)"', f.read(), flags=re.M):
+                if os.path.exists(os.path.join(build_lib.CSRC, inc)):
+                    todo.append(inc)
+    assert seen <= set(build_lib.ATTENTION_SOURCES), seen - set(build_lib.ATTENTION_SOURCES)
