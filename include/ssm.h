@@ -31,6 +31,11 @@
  *     synchronises the stream and returns (and clears) that code.
  *   - Tensors are dense, row-major, with the innermost dimension last, in the
  *     layouts given per argument.  bf16 data are IEEE bfloat16 bit patterns.
+ *   - The library looks up the device addresses of its own device variables
+ *     (the error word, ssm_unmask_noalloc's scratch) once per device and keeps
+ *     them.  Destroying a device's primary context (cudaDeviceReset) makes those
+ *     addresses stale: after a reset, reload the library (a new process) before
+ *     calling it again on that device.
  */
 #ifndef SSM_H_
 #define SSM_H_
@@ -331,6 +336,8 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
  *     return SSM_ERR_CAPACITY and enqueue nothing.
  *   - The first call on a device looks up the array's device address (with
  *     that device current); make that first call before any stream capture.
+ *     The address is kept for the life of the process: a cudaDeviceReset makes
+ *     it stale, so after a reset reload the library before calling this again.
  *   - Every call shares the one array: two calls that overlap on the GPU (on
  *     different streams, or from different threads) race and corrupt each
  *     other's results.  Serialise them.  The array keeps the last call's

@@ -48,7 +48,14 @@ def _digest() -> str:
 
 # The files the attention forward kernel is compiled from (its translation unit and the
 # headers it includes): a change in any of them is a new kernel version.
-ATTENTION_SOURCES = ("attention.cu", "attn_common.cuh", "sm100_ptx.cuh", "tmem_io.cuh", "rope.cuh", "common.cuh")
+ATTENTION_SOURCES = ("attention.cu", "attn_common.cuh", "sm100_ptx.cuh", "tmem_io.cuh", "rope.cuh", "common.cuh",
+                     "ssm.h")
+
+
+def source_path(name: str) -> str:
+    """Path of a kernel source or header: the package's csrc/ first, then include/."""
+    p = os.path.join(CSRC, name)
+    return p if os.path.exists(p) else os.path.join(INCLUDE, name)
 
 
 def source_digest(*names: str) -> str:
@@ -56,7 +63,7 @@ def source_digest(*names: str) -> str:
     to a kernel version)."""
     h = hashlib.sha256()
     for name in names:
-        with open(os.path.join(CSRC, name), "rb") as f:
+        with open(source_path(name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
 

@@ -459,14 +459,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           ++fills;
         }
       }
-      if (!ok) {
-        record_error(p.err, SSM_ERR_TIMEOUT);
-        // let every copy in flight land before the CTA's shared memory is released:
-        // the newest fill of each stage is the only one that can still be in flight
-        if (!half && qcount > 0) warp_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
-        for (int i = max(0, fills - nst); i < fills; ++i)
-          warp_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
-      }
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+      // Every copy in flight lands before the CTA's shared memory is released, on every
+      // path: the newest fill of each stage is the only one that can still be in flight
+      // (an older fill's stage was refilled only after its EMPTY phase, i.e. after it had
+      // landed and been consumed).  A consumer that timed out may have left this warp's last
+      // fills unconsumed even when this warp itself finished; in a run without timeouts they
+      // have all landed and each test below passes at once.  The bound is fixed (kDrainNs),
+      // not the wait limit, which a caller may have shortened.
+      if (!half && qcount > 0) warp_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
+      for (int i = max(0, fills - nst); i < fills; ++i)
+        warp_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
     } else if (warp == 1) {
       // ------------------------------------------------------------- MMA issuer
       bool ok = true;

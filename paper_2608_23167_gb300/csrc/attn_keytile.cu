@@ -279,13 +279,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_keytile_kernel(
           ++fills;
         }
       }
-      if (!ok) {
-        record_error(p.err, SSM_ERR_TIMEOUT);
-        // let every copy in flight land before the CTA's shared memory is released
-        if (!half && qcount > 0) warp_wait(&bars[KT_Q_FULL], (qcount - 1) & 1, kDrainNs);
-        for (int i = max(0, fills - kKtStages); i < fills; ++i)
-          warp_wait(&bars[(half ? KT_V_FULL : KT_K_FULL) + i % kKtStages], (i / kKtStages) & 1, kDrainNs);
-      }
+      if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
+      // every copy in flight lands before the CTA's shared memory is released, on every path
+      // (a consumer that timed out may have left this warp's last fills unconsumed)
+      if (!half && qcount > 0) warp_wait(&bars[KT_Q_FULL], (qcount - 1) & 1, kDrainNs);
+      for (int i = max(0, fills - kKtStages); i < fills; ++i)
+        warp_wait(&bars[(half ? KT_V_FULL : KT_K_FULL) + i % kKtStages], (i / kKtStages) & 1, kDrainNs);
     } else if (warp == 1) {
       // ------------------------------------------------------------- MMA issuer
       bool ok = true;

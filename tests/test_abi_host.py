@@ -119,8 +119,10 @@ def test_attention_digest_covers_its_includes():
         if name in seen:
             continue
         seen.add(name)
-        with open(os.path.join(build_lib.CSRC, name)) as f:
+        with open(build_lib.source_path(name)) as f:
             for inc in re.findall(r'^#include "([^"]+)"', f.read(), flags=re.M):
-                if os.path.exists(os.path.join(build_lib.CSRC, inc)):
-                    todo.append(inc)
+                # every quoted include is a local file of the package or of include/: fail on any
+                # the digest could not read
+                assert os.path.exists(build_lib.source_path(inc)), f"{name} includes unknown {inc}"
+                todo.append(inc)
     assert seen <= set(build_lib.ATTENTION_SOURCES), seen - set(build_lib.ATTENTION_SOURCES)

@@ -2,9 +2,11 @@
 
 Bars: argmax bit-exact (it compares input values only, so it is exact even
 where probabilities are close); conf and p2 within 1e-5 relative of the fp64
-oracle; commits bit-exact for every position whose decision is not within
-rounding of the threshold (|score - threshold| > 1e-5) and, for the
-confidence ranking, where the competing confidences differ by more than 1e-3.
+oracle; commits compared position by position with the oracle's, except for a
+score within 1e-5 of the threshold and for swaps among positions whose
+confidences lie within 1e-3 of the ranking boundary (top-k, min-commit
+fallback) -- see _check_commits.  The separated-confidence cases leave no such
+ambiguity and are compared exactly in every row.
 """
 import numpy as np
 import pytest
@@ -38,35 +40,58 @@ def _gpu_unmask(dev, logits, masked, mode, threshold, topk, min_commit):
     return conf.cpu().double().numpy(), arg.cpu().numpy(), p2.cpu().double().numpy(), commit.cpu().numpy()
 
 
+RANK_TOL = 1e-3      # confidences closer than this may rank either way at fp32
+THRESH_TOL = 1e-5    # a score this close to the threshold may pass either way at fp32
+
+
 def _check_commits(conf_r, p2_r, masked, commit_g, commit_r, mode, threshold, topk, min_commit):
+    """Element-wise commit parity against the oracle, one batch row at a time.
+
+    The rule has two decisions.  (1) Threshold / margin: position j passes if its score
+    (conf, or conf - p2) is above the threshold; GPU and oracle must agree on every
+    position except those whose score is within THRESH_TOL of the threshold.  (2) The
+    ranking: top-k mode commits the k most confident masked positions, and the min-commit
+    fallback adds the most confident non-passing positions.  The GPU's pick must equal the
+    oracle's except for swaps among positions whose oracle confidence lies within RANK_TOL
+    of the decision boundary: no position the GPU left out may be more than RANK_TOL more
+    confident than a position it picked.  Where the boundary pair (the last picked and the
+    first left out) is more than RANK_TOL apart, that makes the pick exactly the oracle's.
+    Returns the number of rows whose commits were compared exactly."""
     batch, B = conf_r.shape
+    exact_rows = 0
     for b in range(batch):
         cand = [j for j in range(B) if masked[b, j]]
-        score = conf_r[b] if mode != O.MODE_MARGIN else conf_r[b] - p2_r[b]
-        ambiguous = False
-        if mode != O.MODE_TOPK:
-            ambiguous = any(abs(score[j] - threshold) <= 1e-5 for j in cand)
-        confs = sorted((conf_r[b, j] for j in cand), reverse=True)
-        if any(abs(confs[i] - confs[i + 1]) <= 1e-3 for i in range(len(confs) - 1)):
-            # the ranking part of the rule is not unique at this precision: check validity only
-            if mode == O.MODE_TOPK:
-                assert commit_g[b].sum() == min(topk, len(cand))
-                continue
-            ambiguous_rank = True
+        got = {j for j in range(B) if commit_g[b, j]}
+        assert got <= set(cand), f"row {b}: commit outside the masked positions"
+        if mode == O.MODE_TOPK:
+            passing, undecided, short = set(), set(), topk
         else:
-            ambiguous_rank = False
-        if ambiguous:
+            score = conf_r[b] if mode == O.MODE_THRESHOLD else conf_r[b] - p2_r[b]
+            passing = {j for j in cand if score[j] > threshold + THRESH_TOL}
+            undecided = {j for j in cand if abs(score[j] - threshold) <= THRESH_TOL}
+            short = min_commit - len(passing)
+        assert passing <= got, f"row {b}: a passing position was not committed"
+        if undecided:
+            # the GPU's passing set is one of the sets between `passing` and `passing | undecided`:
+            # every clearly failing position it commits must come from the fallback
+            extra = got - passing - undecided
+            assert len(extra) <= max(0, min_commit - len(passing)), f"row {b}"
             continue
-        passing = {j for j in cand if score[j] > threshold}
-        if mode != O.MODE_TOPK and not ambiguous_rank:
-            assert commit_g[b].tolist() == commit_r[b].tolist(), b
-        elif mode != O.MODE_TOPK:
-            # every passing position committed; the count follows the min-commit rule
-            assert all(commit_g[b, j] for j in passing)
-            assert commit_g[b].sum() == max(len(passing), min(min_commit, len(cand)))
-        else:
-            assert commit_g[b].tolist() == commit_r[b].tolist(), b
-        assert all(commit_g[b, j] == 0 for j in range(B) if not masked[b, j])
+        rest = [j for j in cand if j not in passing]
+        want = max(0, min(short, len(rest)))
+        picked = got - passing
+        assert len(picked) == want, f"row {b}: {len(picked)} picked by rank, expected {want}"
+        left = [j for j in rest if j not in picked]
+        if picked and left:
+            worst_in = min(conf_r[b, j] for j in picked)
+            best_out = max(conf_r[b, j] for j in left)
+            assert best_out <= worst_in + RANK_TOL, f"row {b}: skipped a position {best_out - worst_in:.2e} more confident"
+        ranked = sorted(rest, key=lambda j: (-conf_r[b, j], j))
+        separated = want == 0 or want == len(ranked) or conf_r[b, ranked[want - 1]] - conf_r[b, ranked[want]] > RANK_TOL
+        if separated:
+            assert commit_g[b].tolist() == commit_r[b].tolist(), f"row {b}"
+            exact_rows += 1
+    return exact_rows
 
 
 @pytest.mark.parametrize("dtype,V,batch,sigma,planted,masked_frac", [
@@ -108,3 +133,50 @@ def test_unmask_ties_and_uniform_rows(dev):
     assert arg[0, 1] == 7 and abs(p2[0, 1] - conf[0, 1]) < 1e-9
     assert arg[0, 2] == V - 1
     assert commit[0].sum() == 1 and commit[0, 1] == 1      # min-1: the most confident row
+
+
+def _separated_logits(batch, B, V, dtype, seed, conf_lo, conf_hi):
+    """N(0, 1) logits in which every position's top id is planted so that its confidence is a
+    target from linspace(conf_lo, conf_hi, B), permuted per row: the confidences of one row are
+    ~(conf_hi - conf_lo) / B apart, far more than RANK_TOL, so every ranking decision is exact."""
+    x = W.draw_logits((batch, B, V), dtype, 1.0, seed)
+    g = torch.Generator().manual_seed(seed + 1)
+    xd = f64(x)
+    targets = np.linspace(conf_lo, conf_hi, B)
+    for b in range(batch):
+        perm = torch.randperm(B, generator=g).numpy()
+        ids = torch.randint(0, V, (B,), generator=g).numpy()
+        for j in range(B):
+            row = xd[b, j]
+            z_rest = np.exp(row).sum() - np.exp(row[ids[j]])
+            c = targets[perm[j]]
+            x[b, j, ids[j]] = float(np.log(c / (1.0 - c) * z_rest))
+    return x
+
+
+@pytest.mark.parametrize("mode,threshold,topk,min_commit", [
+    ("topk", 0.0, 1, 0),            # Vanilla top-1
+    ("topk", 0.0, 3, 0),
+    ("threshold", 0.9, 1, 1),       # nothing above the threshold: the min-1 fallback picks one position
+    ("threshold", 0.9, 1, 2),
+    ("margin", 0.9, 1, 1),
+    ("threshold", 0.5, 1, 1),       # some positions pass, the fallback does not fire
+])
+def test_unmask_commit_positions_separated(dev, mode, threshold, topk, min_commit):
+    """LLaDA vocabulary (126464, bf16), four sequences, confidences planted well apart (0.05 ..
+    0.85): the committed positions are compared with the oracle's in every row, so a kernel that
+    commits the wrong positions (top-k, or the fallback's choice) fails."""
+    batch, B, V = 4, 32, W.LLADA_VOCAB
+    logits = _separated_logits(batch, B, V, "bf16", 31 + topk + min_commit, 0.05, 0.85)
+    g = torch.Generator().manual_seed(5)
+    masked = (torch.rand((batch, B), generator=g) < 0.75).to(torch.uint8)
+    masked[:, 0] = 1
+    md = MODES[mode]
+    conf, arg, p2, commit = _gpu_unmask(dev, logits, masked, md, threshold, topk, min_commit)
+    conf_r, arg_r, p2_r, commit_r = O.unmask(f64(logits), masked.numpy(), md, threshold, topk, min_commit)
+    m = masked.numpy().astype(bool)
+    assert np.array_equal(arg[m], arg_r[m])
+    assert np.allclose(conf[m], conf_r[m], rtol=1e-5, atol=0)
+    exact = _check_commits(conf_r, p2_r, masked.numpy(), commit, commit_r, md, threshold, topk, min_commit)
+    assert exact == batch
+    assert np.array_equal(commit, commit_r)
