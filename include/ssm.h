@@ -273,22 +273,6 @@ ssm_status ssm_attention_varlen_core(const void* q, const void* k_new, const voi
                                      void* out, float* lse, void* workspace, size_t ws_bytes,
                                      ssm_stream_t stream);
 
-/* Which attention forward kernel ssm_attention and ssm_attention_varlen run
- * (process-wide setting; both kernels compute the same function and differ
- * only in how the work is laid on the tensor core):
- *   SSM_ATTN_AUTO         (default) query tiles;
- *   SSM_ATTN_QUERY_TILES  128 query rows (query x head-in-group) per MMA tile
- *                         on the M dimension; any supported shape;
- *   SSM_ATTN_KEY_TILES    128 keys per MMA tile on the M dimension, the query
- *                         rows of one (problem, kv head) on the N dimension in
- *                         multiples of 16 (less padding for short query sets);
- *                         head_dim 128 and max_n_new * (h_q / h_kv) <= 192,
- *                         other calls return SSM_ERR_UNSUPPORTED.
- * Returns SSM_ERR_INVALID_ARG for any other value.  Not synchronised with calls
- * in flight on other host threads. */
-enum { SSM_ATTN_AUTO = 0, SSM_ATTN_QUERY_TILES = 1, SSM_ATTN_KEY_TILES = 2 };
-ssm_status ssm_set_attention_variant(int32_t variant);
-
 /* ------------------------------------------------------------------------- */
 /* 4. Confidence-based unmasking (Sec. 4.2 "Baselines": Vanilla top-1 and     */
 /*    parallel threshold decoding; Sec. 4.6: margin decoding).                */

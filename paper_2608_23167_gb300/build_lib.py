@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libssm.so")
-SOURCES = ["api.cu", "select.cu", "build_input.cu", "unmask.cu", "attention.cu", "attn_keytile.cu", "cache.cu", "topk.cu", "eos.cu"]
+SOURCES = ["api.cu", "select.cu", "build_input.cu", "unmask.cu", "attention.cu", "cache.cu", "topk.cu", "eos.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xptxas", "-v"]

@@ -886,10 +886,6 @@ WsLayout ws_layout(int64_t total_new, int32_t h_q, int32_t h_kv, int32_t d) {
   return l;
 }
 
-std::atomic<int> g_attention_variant{SSM_ATTN_AUTO};
-
-int attention_variant() { return g_attention_variant.load(); }
-
 // One instantiation of the forward: the register split assumes the compiled register count
 // (checked once), the dynamic shared memory is opted into once per device.
 template <int D, bool PACKABLE>
@@ -933,12 +929,6 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   const WsLayout wl = ws_layout(total_new, h_q, h_kv, D);
   auto* qhat = static_cast<__nv_bfloat16*>(workspace);
   auto* khat = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(workspace) + wl.khat);
-  // which kernel: 128-row query tiles unless key tiles (queries on the MMA N dimension)
-  // are requested and every (problem, kv head) has at most kKtMaxRows query rows
-  const bool kt_fits = D == 128 && static_cast<int64_t>(max_n_new) * grp <= kKtMaxRows;
-  const int variant = attention_variant();
-  if (variant == SSM_ATTN_KEY_TILES && !kt_fits) return SSM_ERR_UNSUPPORTED;
-  const bool use_kt = kt_fits && variant == SSM_ATTN_KEY_TILES;
   AttnMaps m;
   {
     const uint64_t dq[3] = {static_cast<uint64_t>(D),
@@ -946,8 +936,6 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                             static_cast<uint64_t>(uniform ? nb * h_kv : 1)};
     const uint32_t bq[3] = {64, kBM, 1};
     if (!make_map(&m.q128, qhat, 3, dq, bq)) return SSM_ERR_CUDA;
-    const uint32_t bq96[3] = {64, 96, 1};
-    if (!make_map(&m.q96, qhat, 3, dq, bq96)) return SSM_ERR_CUDA;
     const uint32_t bkv[4] = {64, 1, kSub, 1};
     const uint64_t dn[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(h_kv),
                             static_cast<uint64_t>(new_rows_per_b), static_cast<uint64_t>(nb)};
@@ -982,7 +970,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   // Packed units need every problem to read one shared cache; a cache too small to hold two of
   // the longest prefixes (or no cache at all) is the only candidate.  Other batches run the
   // forward compiled without packed units, and the pre-pass makes no plan for them.
-  const bool may_pack = !uniform && !use_kt && batch_or_np >= 2 &&
+  const bool may_pack = !uniform && batch_or_np >= 2 &&
                         (cache_rows_per_b == 0 || 2 * static_cast<int64_t>(max_n_cache) > cache_rows_per_b);
   p.plan = may_pack ? reinterpret_cast<AttnPlanHdr*>(static_cast<uint8_t*>(workspace) + wl.plan) : nullptr;
   p.row_prob = may_pack ? reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob) : nullptr;
@@ -1002,13 +990,6 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
                                                           khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK || part == kPartRotate) return s;
-  }
-  if (use_kt) {
-    p.units_per_pg = 1;
-    const int64_t total_units = static_cast<int64_t>(n_prob) * h_kv;
-    if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
-    p.total_units = static_cast<int32_t>(total_units);
-    return launch_attn_keytile(m, p, static_cast<int>(std::min<int64_t>(total_units, num_sms())), st);
   }
   const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
   p.units_per_pg = (m_tiles + 1) / 2;
@@ -1038,13 +1019,6 @@ ssm_status check_attn(const void* q, const void* k_new, const void* v_new, const
 }  // namespace ssm
 
 extern "C" {
-
-ssm_status ssm_set_attention_variant(int32_t variant) {
-  if (variant != SSM_ATTN_AUTO && variant != SSM_ATTN_QUERY_TILES && variant != SSM_ATTN_KEY_TILES)
-    return SSM_ERR_INVALID_ARG;
-  ssm::g_attention_variant.store(variant);
-  return SSM_OK;
-}
 
 size_t ssm_attention_workspace_size(int64_t total_new_rows, int32_t h_q, int32_t h_kv, int32_t head_dim) {
   if (total_new_rows <= 0 || h_q <= 0 || h_kv <= 0 || head_dim <= 0) return 0;

@@ -1,7 +1,6 @@
-// attn_common.cuh -- pieces shared by the two attention forward kernels
-// (attention.cu: 128-row query tiles; attn_keytile.cu: 128-key tiles with the
-// queries on the MMA N dimension): tile constants, the launch parameters, the
-// per-problem geometry, key-tile validity and the warp-level barrier helpers.
+// attn_common.cuh -- pieces of the attention forward (attention.cu): tile
+// constants, the launch parameters, the per-problem geometry, key-tile validity
+// and the warp-level barrier helpers.
 #pragma once
 
 #include <cuda.h>
@@ -164,20 +163,10 @@ __device__ __forceinline__ void warp_arrive(uint64_t* bar) {
   mbar_arrive_if((threadIdx.x & 31) == 0, bar);
 }
 
-// The tensor maps both kernels read: queries packed by GQA group (boxes of 128
-// and of 96 rows), and the cache / new-row keys and values in 32-row and
-// 128-row boxes.
+// The tensor maps the forward reads: queries packed by GQA group (128-row boxes),
+// and the cache / new-row keys and values in 32-row and 128-row boxes.
 struct AttnMaps {
-  CUtensorMap q128, q96, kc, vc, kn, vn, kc128, vc128, kn128, vn128;
+  CUtensorMap q128, kc, vc, kn, vn, kc128, vc128, kn128, vn128;
 };
-
-// Largest number of rows (query x head-in-group) of one (problem, kv head)
-// the key-tile kernel takes; up to kKtSplitKeysMax rows its two softmax slots
-// share the queries and split the key tiles.
-constexpr int kKtMaxRows = 192;
-constexpr int kKtSplitKeysMax = 128;
-
-// Launches attn_keytile_kernel (head_dim 128) on `grid` CTAs.
-ssm_status launch_attn_keytile(const AttnMaps& maps, const AttnParams& p, int grid, cudaStream_t st);
 
 }  // namespace ssm

@@ -65,7 +65,6 @@ def lib() -> ctypes.CDLL:
             "ssm_version": (ctypes.c_char_p, []),
             "ssm_get_device_error": (ctypes.c_int, [vp]),
             "ssm_set_wait_limit_ns": (ctypes.c_int, [ctypes.c_uint64]),
-            "ssm_set_attention_variant": (ctypes.c_int, [i32]),
             "ssm_suffix_count": (ctypes.c_int, [P(SuffixCfg), P(i32), P(i32), P(i32)]),
             "ssm_select_suffix": (ctypes.c_int, [P(SuffixCfg), vp, i32, P(i32), vp]),
             "ssm_select_suffix_batch": (ctypes.c_int, [P(SuffixCfg), i32, vp, i64, P(i64), vp]),
@@ -101,7 +100,6 @@ def lib() -> ctypes.CDLL:
 
 def exported_symbols() -> Sequence[str]:
     return ["ssm_status_str", "ssm_version", "ssm_get_device_error", "ssm_set_wait_limit_ns",
-            "ssm_set_attention_variant",
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
             "ssm_attention_varlen", "ssm_attention_varlen_rotate", "ssm_attention_varlen_core",
@@ -145,14 +143,6 @@ def ssm_set_wait_limit_ns(ns: int) -> None:
 
 
 # ------------------------------------------------------------------------------ selector
-
-
-SSM_ATTN_AUTO, SSM_ATTN_QUERY_TILES, SSM_ATTN_KEY_TILES = 0, 1, 2
-
-
-def ssm_set_attention_variant(variant: int) -> None:
-    """Select the attention kernel for later calls (process-wide; see include/ssm.h)."""
-    _check("ssm_set_attention_variant", lib().ssm_set_attention_variant(int(variant)))
 
 
 def ssm_suffix_count(prompt_len, gen_len, block_len, block_idx, local_budget, middle_budget, tail_budget):

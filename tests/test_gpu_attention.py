@@ -21,21 +21,6 @@ def dev():
     return cuda_or_skip()
 
 
-@pytest.fixture(params=["auto", "query_tiles", "key_tiles"])
-def variant(request, dev):
-    """Runs a test under each attention kernel (include/ssm.h: ssm_set_attention_variant)."""
-    from paper_2608_23167_gb300 import ssm
-    code = {"auto": ssm.SSM_ATTN_AUTO, "query_tiles": ssm.SSM_ATTN_QUERY_TILES,
-            "key_tiles": ssm.SSM_ATTN_KEY_TILES}[request.param]
-    ssm.ssm_set_attention_variant(code)
-    yield request.param
-    ssm.ssm_set_attention_variant(ssm.SSM_ATTN_AUTO)
-
-
-def _key_tiles_fit(n_new, h_q, h_kv, d):
-    return d == 128 and n_new * (h_q // h_kv) <= 192
-
-
 def _ramp(t: torch.Tensor, top: float) -> torch.Tensor:
     """Scales row i of [batch, rows, h, d] by 1 + (top - 1) i / rows: later keys score higher,
     so the running maximum keeps growing past the first key tile (the lazy rescale path)."""
@@ -72,34 +57,29 @@ def _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed, pos=None, with_l
     (1, 73, 64, 4, 4, 64, 1e4, 0),          # tiny workload (b = 0)
     (1, 589, 0, 8, 8, 128, 5e5, 0),         # LLaDA no-cache shape (8 of 32 heads), 5 query tiles
     (2, 132, 512, 14, 2, 128, 1e6, 0),      # Dream GQA, 7 query heads per kv head
-    (2, 101, 512, 8, 8, 128, 5e5, 0),       # serving shape (8 of 32 heads); key tiles: keys split, N = 112
+    (2, 101, 512, 8, 8, 128, 5e5, 0),       # serving shape (8 of 32 heads): one query tile, keys split
     (1, 1, 0, 2, 1, 64, 1e4, 0),            # a single key
     (3, 37, 100, 4, 2, 128, 0.0, 0),        # ragged cache (100 = 3*32 + 4), no rotary encoding
     (1, 200, 1000, 2, 2, 64, 1e4, 0),       # cache and new segments both ragged
-    (1, 129, 31, 4, 4, 128, 5e5, 0),        # one row past a query tile; key tiles: queries split 80 + 64
-    (1, 172, 1024, 4, 4, 128, 5e5, 0),      # long sweep at block 0; key tiles: queries split 96 + 80
-    (1, 96, 65, 4, 2, 128, 1e4, 0),         # GQA, 192 rows: the key-tile maximum, queries split 96 + 96
-    (1, 128, 77, 2, 2, 128, 1e4, 0),        # 128 rows: the largest keys-split unit (N = 128)
-    (2, 16, 300, 2, 1, 128, 1e4, 0),        # 32 rows, N = 32
-    (1, 5, 0, 2, 2, 128, 1e4, 0),           # one key tile: slot B of a keys-split unit has no work, N = 16
+    (1, 129, 31, 4, 4, 128, 5e5, 0),        # one row past a query tile: a second tile of one row
+    (1, 172, 1024, 4, 4, 128, 5e5, 0),      # long sweep at block 0
+    (1, 96, 65, 4, 2, 128, 1e4, 0),         # GQA, 192 rows in two query tiles
+    (1, 128, 77, 2, 2, 128, 1e4, 0),        # 128 rows: the largest keys-split unit
+    (2, 16, 300, 2, 1, 128, 1e4, 0),        # 32 rows
+    (1, 5, 0, 2, 2, 128, 1e4, 0),           # one key tile: slot B of a keys-split unit has no work
     (1, 150, 900, 2, 2, 128, 0.0, 4.0),     # cache keys ramped x1..x4: maxima grow past the first tile
     (1, 100, 900, 2, 2, 128, 0.0, 4.0),     # the same with the keys split between the slots
     (1, 150, 900, 2, 2, 128, 0.0, 16.0),    # x1..x16: later tiles' p reach 2^50 against the first tile's
     (1, 100, 900, 2, 2, 128, 0.0, 16.0),    #   maximum, so the exact (rescaling) path runs, both layouts
 ])
-def test_attention_matches_oracle(dev, variant, batch, n_new, n_cache, h_q, h_kv, d, theta, ramp):
+def test_attention_matches_oracle(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, ramp):
     from paper_2608_23167_gb300 import ssm
-    if variant == "key_tiles" and not _key_tiles_fit(n_new, h_q, h_kv, d):
-        with pytest.raises(ssm.SSMError) as e:
-            _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache, ramp=ramp)
-        assert e.value.status == ssm.SSM_ERR_UNSUPPORTED
-        return
     out, ref, lse, ref_lse = _run(dev, batch, n_new, n_cache, h_q, h_kv, d, theta, seed=n_new + n_cache, ramp=ramp)
-    assert_attention_close(out, ref, f"{variant} b{batch} n{n_new} c{n_cache} h{h_q}/{h_kv} d{d}")
+    assert_attention_close(out, ref, f"b{batch} n{n_new} c{n_cache} h{h_q}/{h_kv} d{d}")
     assert np.abs(lse - ref_lse).max() <= 2e-2
 
 
-def test_attention_full_workloads_sampled(dev, variant):
+def test_attention_full_workloads_sampled(dev):
     """Full-size serving and Dream launches; the oracle checks a sample of heads."""
     from paper_2608_23167_gb300 import ssm
     for name in ("serve", "dream"):
@@ -114,8 +94,6 @@ def test_attention_full_workloads_sampled(dev, variant):
         kc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 34)
         vc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 35)
         o = torch.empty((w.batch, n_new, w.h_q, w.head_dim), dtype=torch.bfloat16, device=dev)
-        if variant == "key_tiles" and not _key_tiles_fit(n_new, w.h_q, w.h_kv, w.head_dim):
-            continue
         ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), o, w.rope_theta)
         torch.cuda.synchronize()
         check_device_error()
@@ -129,7 +107,7 @@ def test_attention_full_workloads_sampled(dev, variant):
             assert_attention_close(f64(o[b:b + 1, :, hs]), ref, f"{name} batch {b}")
 
 
-def test_attention_varlen_block_sweep(dev, variant):
+def test_attention_varlen_block_sweep(dev):
     """The long-sequence sweep: every block index 0..63 as one ragged launch over a
     shared prefix cache; the oracle checks several block indices on a few heads."""
     from paper_2608_23167_gb300 import ssm
@@ -168,7 +146,7 @@ def test_attention_varlen_block_sweep(dev, variant):
         assert np.abs(lg[sl][None] - ref_lse).max() <= 2e-2
 
 
-def test_attention_key_permutation_invariance(dev, variant):
+def test_attention_key_permutation_invariance(dev):
     """Permuting the new rows together with their positions permutes the output rows."""
     from paper_2608_23167_gb300 import ssm
     n, c, h, d = 150, 70, 4, 128
@@ -257,7 +235,7 @@ def test_attention_varlen_serving_batch(dev):
 
 
 @pytest.mark.parametrize("shape", ["llada", "serve"])
-def test_attention_varlen_cold_l2_and_graph_replay(dev, variant, shape):
+def test_attention_varlen_cold_l2_and_graph_replay(dev, shape):
     """Pipeline timing edge cases: every launch behind a 256 MB write (cold L2, slow tile loads
     while the producers run ahead), eagerly and as CUDA-graph replays, with a 0.2 s wait limit so
     a stuck barrier wait reports SSM_ERR_TIMEOUT quickly; the outputs must equal a warm launch's.
@@ -269,8 +247,6 @@ def test_attention_varlen_cold_l2_and_graph_replay(dev, variant, shape):
         sizes, cache_rows = [(589, 0)], 0
     else:
         sizes, cache_rows = [(101, 512)] * 8, 8 * 512
-    if variant == "key_tiles" and not _key_tiles_fit(max(n for n, _ in sizes), h, h, d):
-        pytest.skip("shape outside the key-tile kernel")
     rows, new_row = [], 0
     for i, (n, c) in enumerate(sizes):
         rows.append((new_row, i * c, n, c))
@@ -313,7 +289,7 @@ def test_attention_varlen_cold_l2_and_graph_replay(dev, variant, shape):
 
 
 @pytest.mark.parametrize("case", ["mixed", "gqa", "d64", "one_row"])
-def test_attention_varlen_packed_prefix(dev, variant, case):
+def test_attention_varlen_packed_prefix(dev, case):
     """Ragged batches whose problems read prefixes of one shared cache and whose new rows
     follow one another: the kernel packs the rows of consecutive problems into shared query
     tiles (each row masked to its own prefix and its own new rows).  Every problem is checked
@@ -332,8 +308,6 @@ def test_attention_varlen_packed_prefix(dev, variant, case):
         sizes = [(37, 100), (1, 0), (130, 250), (64, 250), (5, 31), (200, 512), (33, 64)]
     else:
         sizes = [(1, (7 * i) % 200) for i in range(300)]
-    if variant == "key_tiles" and not _key_tiles_fit(max(n for n, _ in sizes), h_q, h_kv, d):
-        pytest.skip("shape outside the key-tile kernel")
     cache_rows = max(c for _, c in sizes) or 1
     rows, new_row = [], 0
     for n, c in sizes:
