@@ -653,10 +653,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           for (int s4 = 0; s4 < 4; ++s4) lo[s4] = 0;
         }
         const bool full_tile = __all_sync(0xffffffffu, full_row);
-        // this row's scores of the tile, invalid keys at -inf (selects, no branch per row)
-        auto load_s = [&]() {
+        // A row sees all keys of most sub-boxes or none of them (a whole sub-box of another
+        // problem's new rows, or of cache rows past its prefix): the exponent's addend carries
+        // that (-inf: none), with no per-key work.  Only when some row of the warp sees part of
+        // a sub-box (one vote, warp-uniform) are the invalid keys set to -inf one by one; a row
+        // maximum (first tile of a unit, exact path) takes them all masked.
+        bool whole = true;
+#pragma unroll
+        for (int s4 = 0; s4 < 4; ++s4) whole = whole && ((lo[s4] == 0 && hi[s4] == kSub) || hi[s4] <= lo[s4]);
+        const bool part_keys = !__all_sync(0xffffffffu, whole);
+        auto load_s = [&](bool for_max) {
           tmem_ld_x128(tS, sr);
-          if (!full_tile) {
+          if (for_max ? !full_tile : part_keys) {
 #pragma unroll
             for (int c = 0; c < kBN; ++c) {
               const int cc = c & (kSub - 1);
@@ -664,7 +672,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
             }
           }
         };
-        load_s();
+        load_s(k == 0);
         const float sc = p.scale_log2;
         // row maximum of the tile's scores: eight independent chains of 3-input max, then a short tree
         auto row_max = [&]() -> float {
@@ -680,12 +688,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         // pair sums; returns the row's sum of p over the tile
         uint32_t pk[kBN / 2];
         auto exp_pass = [&](float m) -> float {
-          const float neg = -m;
+          float add[4];
+#pragma unroll
+          for (int s4 = 0; s4 < 4; ++s4) add[s4] = hi[s4] <= lo[s4] ? -INFINITY : -m;
           float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int c = 0; c < kBN / 2; ++c) {
             float t0, t1;
-            ffma2(t0, t1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), sc, sc, neg, neg);
+            const float a0 = add[c / (kSub / 2)];
+            ffma2(t0, t1, __uint_as_float(sr[2 * c]), __uint_as_float(sr[2 * c + 1]), sc, sc, a0, a0);
             const float a = ex2_approx(t0), b = ex2_approx(t1);
             fadd2_acc(ra[c & 3], rb[c & 3], a, b);
             pk[c] = pack_bf16x2(a, b);
@@ -710,7 +721,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           if (__any_sync(0xffffffffu, need)) {
             // S is still in tensor memory (P has not been written over it): load it again
             // rather than keep the scores live through the exponentials
-            load_s();
+            load_s(true);
             const float m_new = fmaxf(m_run, row_max() * sc);
             const float alpha = ex2_approx(need ? m_run - m_new : 0.f);
             // the previous PV of this slot completed before this S tile was committed
@@ -771,15 +782,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const float inv = 1.f / lsum;
         const float ca = a * inv, cb = b * inv;
         __nv_bfloat16* dst = p.out + (qrow * p.h_q + h) * D;
-        // 32 output columns of this row from fp32 values: bf16, four 16-byte stores
+        // 32 output columns of this row from fp32 values: bf16, two 32-byte stores (four 16-byte
+        // ones if the output is only 16-byte aligned).  A warp's rows lie h_q * d apart, so each
+        // store instruction touches 32 lines: wider stores halve the instructions
         auto store32 = [&](int c0, const float (&f)[32]) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c0);
+          uint4 v4[4];
 #pragma unroll
           for (int v = 0; v < 4; ++v)
-            st_global_v4_pred(d4 + v,
-                              make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
-                                         pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7])),
-                              valid);
+            v4[v] = make_uint4(pack_bf16x2(f[8 * v + 0], f[8 * v + 1]), pack_bf16x2(f[8 * v + 2], f[8 * v + 3]),
+                               pack_bf16x2(f[8 * v + 4], f[8 * v + 5]), pack_bf16x2(f[8 * v + 6], f[8 * v + 7]));
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c0);
+          if (p.out_v8) {
+            st_global_v8_pred(d4, v4[0], v4[1], valid);
+            st_global_v8_pred(d4 + 2, v4[2], v4[3], valid);
+          } else {
+#pragma unroll
+            for (int v = 0; v < 4; ++v) st_global_v4_pred(d4 + v, v4[v], valid);
+          }
         };
         if (!w.two && w.nt >= 2) {
           // split keys: both accumulators, 64 columns at a time, each pair of loads one round trip
@@ -976,6 +995,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.row_prob = may_pack ? reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob) : nullptr;
   p.scale_log2 = scale * kLog2e;
   p.out = static_cast<__nv_bfloat16*>(out);
+  p.out_v8 = (reinterpret_cast<uintptr_t>(out) & 31u) == 0 ? 1 : 0;
   p.lse = lse;
   p.err = device_error_word();
   p.wait_ns = wait_limit_ns();

@@ -63,6 +63,7 @@ struct AttnParams {
   int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)
   __nv_bfloat16* out;
+  int32_t out_v8;                    // out is 32-byte aligned: 32-byte epilogue stores
   float* lse;
   unsigned* err;
   uint64_t wait_ns;

@@ -309,6 +309,17 @@ __device__ __forceinline__ void st_global_v4_pred(void* ptr, uint4 v, bool pred)
       : "memory");
 }
 
+// 32-byte store (sm_100+ 256-bit vector form); ptr must be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8_pred(void* ptr, uint4 lo, uint4 hi, bool pred) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.u32 p, %9, 0;\n\t"
+      "@p st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n\t}\n" ::"l"(ptr),
+      "r"(lo.x), "r"(lo.y), "r"(lo.z), "r"(lo.w), "r"(hi.x), "r"(hi.y), "r"(hi.z), "r"(hi.w),
+      "r"(static_cast<uint32_t>(pred))
+      : "memory");
+}
+
 __device__ __forceinline__ void st_global_f32_pred(float* ptr, float v, bool pred) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
