@@ -182,7 +182,7 @@ class StepInputs:
         return float(masked_rows * w.vocab * self.logits.element_size())
 
     # -- one pass of the hot path ---------------------------------------------------------
-    def step(self, ev=None):
+    def step(self, ev=None, unmask=None):
         from paper_2608_23167_gb300 import ssm
         w = self.w
         if ev is not None:
@@ -205,8 +205,11 @@ class StepInputs:
         if ev is not None:
             ev[4].record()
         # the threshold rule needs no second-largest probability, so p2 is not requested
-        ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=None,
-                       threshold=w.threshold, min_commit=1, workspace=self.unmask_ws)
+        if unmask is not None:
+            unmask()
+        else:
+            ssm.ssm_unmask(self.logits, self.masked, self.conf, self.argmax, self.commit, p2=None,
+                           threshold=w.threshold, min_commit=1, workspace=self.unmask_ws)
         if ev is not None:
             ev[5].record()
 
@@ -332,7 +335,7 @@ def time_stages(inp: StepInputs, reps: int, flush) -> np.ndarray:
     """Per-stage device times: each rep enqueues a GPU-side delay, then the step's calls with
     an event between stages, so the host has queued the whole step before the device reaches
     it and no host time falls between two events."""
-    acc = np.zeros(5)
+    rows = []
     for i in range(reps):
         if flush is not None:
             flush.fill_(i & 0x7F)
@@ -340,8 +343,10 @@ def time_stages(inp: StepInputs, reps: int, flush) -> np.ndarray:
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
         inp.step(ev)
         torch.cuda.synchronize()
-        acc += [ev[j].elapsed_time(ev[j + 1]) for j in range(5)]
-    return acc / max(reps, 1)
+        rows.append([ev[j].elapsed_time(ev[j + 1]) for j in range(5)])
+    a = np.array(rows).reshape(-1, 5)
+    time_stages.last_median = np.median(a, axis=0)
+    return a.mean(axis=0)
 
 
 def time_e2e(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
@@ -472,6 +477,7 @@ def stage_report(inp: "StepInputs", stage_ms, step_ms: float, peaks: dict) -> di
         "attn_fwd_ms": core_ms, "attn_fwd_TFLOPs": tf(core_ms),
         "attn_fwd_frac_bf16_burst": tf(core_ms) / burst,
         "attn_fwd_frac_bf16_sustained": tf(core_ms) / sustained,
+        "attn_fwd_ms_median": float(getattr(time_stages, "last_median", [0.0] * 5)[3]),
         "unmask_ms": unmask_ms, "unmask_GBps": gb(inp.unmask_bytes(), unmask_ms),
         "unmask_frac_hbm": gb(inp.unmask_bytes(), unmask_ms) / hbm,
         "unmask_frac_8TBps_nominal": gb(inp.unmask_bytes(), unmask_ms) / 8000.0,
@@ -644,14 +650,29 @@ def time_next_rows(inp: "StepInputs", attn_ms: float, dev, hbm_peak: float, tens
     out["early_stop"] = {"sequences": inp.n, "gen_len": w.gen, "us": ms * 1e3, "bound": "launch latency"}
     del toks, fin, nact
     n = max(inp.total_suffix, 1)
-    lg = W.draw_logits((n, w.vocab), "bf16", w.logits_sigma, 73, device=dev)
+    lg = W.draw_logits((n, w.vocab), inp.w.logits_dtype, w.logits_sigma, 73, device=dev)
     ids = torch.empty((n, w.topk), dtype=torch.int32, device=dev)
     pr = torch.empty((n, w.topk), dtype=torch.float32, device=dev)
     ms = _event_ms(lambda: ssm.ssm_suffix_topk(lg, w.topk, ids, pr), reps=10)
-    nbytes = float(n) * w.vocab * 2
+    nbytes = float(n) * w.vocab * lg.element_size()
     out["suffix_topk"] = {"rows": n, "k": w.topk, "ms": ms, "GBps": nbytes / (ms * 1e-3) / 1e9,
                           "frac_hbm": nbytes / (ms * 1e-3) / 1e9 / hbm_peak,
                           "bytes": "the logits of the retained suffix rows, read once"}
+    # the step with everything the next step needs from the logits: ssm_unmask_topk (block rows'
+    # commits and the retained suffix rows' top-k) in place of ssm_unmask, as graph replays
+    logits_pass = lambda: ssm.ssm_unmask_topk(inp.logits, inp.masked, inp.conf, inp.argmax, inp.commit, lg,  # noqa: E731
+                                              w.topk, ids, pr, threshold=w.threshold, min_commit=1,
+                                              workspace=inp.unmask_ws)
+    ms_lp = _event_ms(logits_pass, reps=10)
+    lp_bytes = inp.unmask_bytes() + nbytes
+    step_ms = _event_ms(lambda: inp.step(unmask=logits_pass), reps=20)
+    out["step_with_suffix_topk"] = {
+        "value": inp.n / (step_ms * 1e-3), "unit": UNIT, "ms_per_step": step_ms,
+        "logits_ms": ms_lp, "logits_GBps": lp_bytes / (ms_lp * 1e-3) / 1e9,
+        "logits_frac_hbm": lp_bytes / (ms_lp * 1e-3) / 1e9 / hbm_peak,
+        "how": "the step (eager calls, back to back) with ssm_unmask_topk over the block rows' and the retained "
+               "suffix rows' logits in place of ssm_unmask; logits_* is that call alone (its bytes: both sets of "
+               "logits, read once)"}
     del lg, ids, pr
     n = 8192
     kn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 71).to(dev)

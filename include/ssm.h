@@ -305,6 +305,25 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
                       int32_t topk, int32_t min_commit, float* conf, int32_t* argmax, float* p2,
                       uint8_t* commit, void* workspace, size_t ws_bytes, ssm_stream_t stream);
 
+/* Everything a denoising step takes from its logits, in one call: ssm_unmask
+ * of the block rows (Sec. 4.2 / 4.6 commit rules) and ssm_suffix_topk of the
+ * retained suffix rows (Sec. 3.2 "Soft Suffix Embedding Mixing": the top-k
+ * candidates and full-vocabulary probabilities that the next step's Eq. 6
+ * renormalizes -- ssm_build_step_input's prev_topk_ids / prev_topk_prob).  The
+ * two streaming passes are enqueued back to back on `stream`.
+ * Block-row arguments, outputs and workspace as ssm_unmask; suffix rows as
+ * ssm_suffix_topk:
+ *   suffix_logits  same dtype and vocab as logits, [n_suffix_rows, vocab]
+ *   ids, probs     int32 / fp32 [n_suffix_rows, k], 1 <= k <= 8
+ * Every condition of both calls is checked before anything is enqueued
+ * (n_suffix_rows == 0 is ssm_unmask).  The results equal the two separate
+ * calls'. */
+ssm_status ssm_unmask_topk(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len, int64_t vocab,
+                           const uint8_t* masked, ssm_commit_mode mode, float threshold, int32_t topk,
+                           int32_t min_commit, float* conf, int32_t* argmax, float* p2, uint8_t* commit,
+                           const void* suffix_logits, int64_t n_suffix_rows, int32_t k, int32_t* ids,
+                           float* probs, void* workspace, size_t ws_bytes, ssm_stream_t stream);
+
 /* ssm_unmask_noalloc -- ssm_unmask for callers that cannot allocate device
  * memory.  The paper has no counterpart: this is a deployment convenience.
  *

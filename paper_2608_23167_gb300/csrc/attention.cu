@@ -320,7 +320,7 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
   return w;
 }
 
-template <int D, bool PACKABLE>
+template <int D, bool PACKABLE, bool POLL>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
     const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kn,
@@ -397,7 +397,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
         if (!half) {
-          if (qcount > 0) ok = warp_wait(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
+          if (qcount > 0) ok = warp_wait<POLL>(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
           if (!ok) break;
           const int nq = w.two ? 2 : 1;
           mbar_arrive_expect_tx_if(leader, &bars[Q_FULL], nq * L::TILE);
@@ -420,7 +420,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const int c3 = uniform ? w.prob : 0;
         for (int jt = 0; jt < w.nt && ok; ++jt) {
           const int st = fills % nst, fill = fills / nst;
-          if (fill > 0) ok = warp_wait(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
+          if (fill > 0) ok = warp_wait<POLL>(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
           if (!ok) break;
           uint64_t* full = &bars[(half ? V_FULL : K_FULL) + st];
           mbar_arrive_expect_tx_if(leader, full, L::TILE);
@@ -467,9 +467,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       // fills unconsumed even when this warp itself finished; in a run without timeouts they
       // have all landed and each test below passes at once.  The bound is fixed (kDrainNs),
       // not the wait limit, which a caller may have shortened.
-      if (!half && qcount > 0) warp_wait(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
+      if (!half && qcount > 0) warp_wait<POLL>(&bars[Q_FULL], (qcount - 1) & 1, kDrainNs);
       for (int i = max(0, fills - nst); i < fills; ++i)
-        warp_wait(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
+        warp_wait<POLL>(&bars[(half ? V_FULL : K_FULL) + i % nst], (i / nst) & 1, kDrainNs);
     } else if (warp == 1) {
       // ------------------------------------------------------------- MMA issuer
       bool ok = true;
@@ -483,7 +483,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
         const Unit w = make_unit(p, up, u);
         if (!w.valid) continue;
-        ok = warp_wait(&bars[Q_FULL], ucount & 1, p.wait_ns);
+        ok = warp_wait<POLL>(&bars[Q_FULL], ucount & 1, p.wait_ns);
         if (!ok) break;
         int kx0 = 0, kx1 = 0;        // jobs issued per slot in this unit
         int jlast0 = 0, jlast1 = 0;  // key tile of each slot's latest QK^T
@@ -493,7 +493,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           bool& f = x ? freed1 : freed0;
           if (f) return true;
           f = true;
-          return ucount == 0 || warp_wait(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
+          return ucount == 0 || warp_wait<POLL>(&bars[O_FREE + x], (ucount - 1) & 1, p.wait_ns);
         };
         // O_X += P_X V(j) for slot X's latest job
         auto issue_pv = [&](int x) -> bool {
@@ -501,7 +501,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           int& pv = x ? pv1 : pv0;
           if (!wait_o_free(x)) return false;
           // the K/V watcher's share of this phase vouches for V(jp) and this slot's next K tile
-          if (!warp_wait(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
+          if (!warp_wait<POLL>(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
           const int vi = vbase + jp;
           tc_fence_after_sync();
           const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
@@ -524,7 +524,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           if ((x ? kx1 : kx0) > 0)
             ok = issue_pv(x);  // the watcher's share of P_FULL vouches for this slot's next K tile too
           else
-            ok = warp_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
+            ok = warp_wait<POLL>(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
           if (!ok) break;
           tc_fence_after_sync();
           const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
@@ -550,7 +550,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
       // every issued MMA completes before tensor memory is released
       umma_commit_if(leader, &bars[DRAIN]);
-      warp_wait(&bars[DRAIN], 0, kDrainNs);
+      warp_wait<POLL>(&bars[DRAIN], 0, kDrainNs);
     } else {
       // ------------------------------------------------------------- K/V watcher (warp 3)
       // Every mbarrier test costs the MMA-issuing warp ~150 cycles in which it issues
@@ -570,18 +570,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       // one arrival for slot x's PV of tile jp
       auto vouch = [&](int x, int jp, int jk) -> bool {
         int& d = x ? done1 : done0;
-        if (d > 0 && !warp_wait(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
+        if (d > 0 && !warp_wait<POLL>(&bars[P_FULL + x], (d - 1) & 1, p.wait_ns)) return false;
         // slot x's d-th QK^T (on K tile jp) has completed, so tile jp has landed; every S
         // of each slot is seen here in order, so the fill before any K tile waited for
         // below is known to have landed (split keys: tile jp itself; both slots on every
         // tile: tile jp - 1, or the previous unit's last tile), and the fill after it
         // needs this vouch: each parity wait stays within its two-phase window
-        if (!warp_wait(&bars[S_FULL + x], d & 1, p.wait_ns)) return false;
+        if (!warp_wait<POLL>(&bars[S_FULL + x], d & 1, p.wait_ns)) return false;
         for (; vconf <= kbase + jp; ++vconf)
-          if (!warp_wait(&bars[V_FULL + vconf % kVStages], (vconf / kVStages) & 1, p.wait_ns)) return false;
+          if (!warp_wait<POLL>(&bars[V_FULL + vconf % kVStages], (vconf / kVStages) & 1, p.wait_ns)) return false;
         if (jk >= 0) {
           const int ki = kbase + jk;
-          if (!warp_wait(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns)) return false;
+          if (!warp_wait<POLL>(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns)) return false;
         }
         mbar_arrive_if(leader, &bars[P_FULL + x]);
         ++d;
@@ -638,7 +638,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       }
       for (int k = 0; k < jobs; ++k) {
         const int j = w.two ? k : 2 * k + x;
-        ok = warp_wait(&bars[S_FULL + x], sj & 1, p.wait_ns);
+        ok = warp_wait<POLL>(&bars[S_FULL + x], sj & 1, p.wait_ns);
         if (!ok) break;
         tc_fence_after_sync();
         uint32_t sr[kBN];
@@ -725,7 +725,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
             const float m_new = fmaxf(m_run, row_max() * sc);
             const float alpha = ex2_approx(need ? m_run - m_new : 0.f);
             // the previous PV of this slot completed before this S tile was committed
-            ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
+            ok = warp_wait<POLL>(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
             if (!ok) break;
             tc_fence_after_sync();
 #pragma unroll
@@ -749,7 +749,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         ++sj;
       }
       // the slot's last PV of this unit (it completes before any later S of this slot)
-      if (ok && jobs > 0) ok = warp_wait(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
+      if (ok && jobs > 0) ok = warp_wait<POLL>(&bars[O_DONE + x], (sj - 1) & 1, p.wait_ns);
       if (!ok) break;
       tc_fence_after_sync();
       // Split keys: slot B hands its (max, sum) to slot A, which merges both accumulators.
@@ -762,7 +762,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           merge_buf[kBM + row] = l_run;
           warp_arrive(&bars[MERGE_FULL]);
         } else {
-          ok = warp_wait(&bars[MERGE_FULL], merges & 1, p.wait_ns);
+          ok = warp_wait<POLL>(&bars[MERGE_FULL], merges & 1, p.wait_ns);
           if (!ok) break;
           mB = merge_buf[row];
           lB = merge_buf[kBM + row];
@@ -907,14 +907,14 @@ WsLayout ws_layout(int64_t total_new, int32_t h_q, int32_t h_kv, int32_t d) {
 
 // One instantiation of the forward: the register split assumes the compiled register count
 // (checked once), the dynamic shared memory is opted into once per device.
-template <int D, bool PACKABLE>
-ssm_status launch_fwd(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
+template <int D, bool PACKABLE, bool POLL>
+ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
   using L = Layout<D>;
   static std::atomic<int> regs_ok{0};  // 0 unknown, 1 ok, 2 mismatch
   int st_regs = regs_ok.load();
   if (st_regs == 0) {
     cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, PACKABLE>) != cudaSuccess) return SSM_ERR_CUDA;
+    if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, PACKABLE, POLL>) != cudaSuccess) return SSM_ERR_CUDA;
     st_regs = fa.numRegs == kLaunchRegs ? 1 : 2;
     regs_ok.store(st_regs);
   }
@@ -924,14 +924,23 @@ ssm_status launch_fwd(const AttnMaps& m, const AttnParams& p, int grid, cudaStre
   if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
   const uint64_t bit = 1ull << (dev & 63);
   if (!(attr_set.load() & bit)) {
-    if (cudaFuncSetAttribute(attn_fwd_kernel<D, PACKABLE>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
+    if (cudaFuncSetAttribute(attn_fwd_kernel<D, PACKABLE, POLL>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
         cudaSuccess)
       return SSM_ERR_CUDA;
     attr_set.fetch_or(bit);
   }
-  attn_fwd_kernel<D, PACKABLE><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
+  attn_fwd_kernel<D, PACKABLE, POLL><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
                                                                      m.kn128, m.vn128, p);
   return launch_status();
+}
+
+// The forward for this call's wait limit: limits below the try_wait suspend window take the
+// form whose waits poll without blocking (so that the limit holds); the usual limits, the
+// form with blocking probes.
+template <int D, bool PACKABLE>
+ssm_status launch_fwd(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
+  if (p.wait_ns < kPollLimitNs) return launch_fwd_form<D, PACKABLE, true>(m, p, grid, st);
+  return launch_fwd_form<D, PACKABLE, false>(m, p, grid, st);
 }
 
 template <int D>

@@ -147,17 +147,22 @@ __device__ __forceinline__ bool tile_valid_counts(int j, int n_csub, int n_nsub,
 // TMEM load issued that way ended a kernel with an unspecified launch failure).
 // So every lane polls the barrier and the loop is steered by warp votes, and the
 // single arrival of a warp is a predicated instruction rather than a branch.
-// The suspend-time hint of each try_wait is the wait limit itself when that is below the
-// default 20 us, so a short limit is honoured from the first probe on.
+// POLL: every probe is the non-blocking test_wait, so the limit is checked between probes
+// whatever it is (a blocking try_wait may sleep until its phase completes, up to its ~20 us
+// suspend window).  The host launches the polling form of a kernel only for wait limits
+// below that window.
+template <bool POLL = false>
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (__all_sync(0xffffffffu, mbar_test_wait(bar, parity))) return true;
   const uint64_t t0 = global_timer_ns();
-  const uint32_t hint = limit_ns < 20000u ? static_cast<uint32_t>(limit_ns) : 20000u;
   while (true) {
-    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity, hint))) return true;
+    if (__all_sync(0xffffffffu, POLL ? mbar_test_wait(bar, parity) : mbar_try_wait(bar, parity))) return true;
     if (__any_sync(0xffffffffu, global_timer_ns() - t0 > limit_ns)) return false;
   }
 }
+
+// Wait limits below this are polled (see warp_wait).
+constexpr uint64_t kPollLimitNs = 20000;
 
 __device__ __forceinline__ void warp_arrive(uint64_t* bar) {
   __syncwarp();

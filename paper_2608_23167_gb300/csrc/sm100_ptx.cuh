@@ -111,9 +111,8 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (mbar_test_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
-  const uint32_t hint = limit_ns < 20000u ? static_cast<uint32_t>(limit_ns) : 20000u;
   while (true) {
-    if (mbar_try_wait(bar, parity, hint)) return true;
+    if (mbar_try_wait(bar, parity)) return true;
     if (global_timer_ns() - t0 > limit_ns) return false;
   }
 }

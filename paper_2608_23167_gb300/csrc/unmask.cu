@@ -1,5 +1,7 @@
 // unmask.cu -- confidence-based unmasking (Sec. 4.2 "Baselines": Vanilla top-1
-// and parallel threshold decoding; Sec. 4.6: margin decoding).
+// and parallel threshold decoding; Sec. 4.6: margin decoding), and
+// ssm_unmask_topk, which also enqueues the retained suffix positions' top-k
+// (topk.cu) for the next step's Eq. 6.
 //
 // Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
 // segments of whole 16 KB chunks (the work items, dealt round-robin to
@@ -25,6 +27,7 @@
 #include "common.cuh"
 #include "sm100_ptx.cuh"
 #include "stream.cuh"
+#include "topk.cuh"
 
 namespace ssm {
 namespace {
@@ -499,6 +502,48 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
                                                          threshold, topk, min_commit, conf, argmax, p2,
                                                          commit);
   return ssm::launch_status();
+}
+
+ssm_status ssm_unmask_topk(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len, int64_t vocab,
+                           const uint8_t* masked, ssm_commit_mode mode, float threshold, int32_t topk,
+                           int32_t min_commit, float* conf, int32_t* argmax, float* p2, uint8_t* commit,
+                           const void* suffix_logits, int64_t n_suffix_rows, int32_t k, int32_t* ids,
+                           float* probs, void* workspace, size_t ws_bytes, ssm_stream_t stream) {
+  if (n_suffix_rows < 0) return SSM_ERR_INVALID_ARG;
+  if (n_suffix_rows == 0)
+    return ssm_unmask(logits, dtype, batch, block_len, vocab, masked, mode, threshold, topk, min_commit, conf,
+                      argmax, p2, commit, workspace, ws_bytes, stream);
+  if (dtype != SSM_DTYPE_BF16 && dtype != SSM_DTYPE_F32) return SSM_ERR_UNSUPPORTED;
+  if (k < 1 || k > 8) return SSM_ERR_UNSUPPORTED;
+  if (vocab <= 0 || k > vocab || !suffix_logits || !ids || !probs) return SSM_ERR_INVALID_ARG;
+  if (batch < 0 || block_len < 0) return SSM_ERR_INVALID_ARG;
+  if (batch == 0 || block_len == 0)
+    return ssm_suffix_topk(suffix_logits, dtype, n_suffix_rows, vocab, k, ids, probs, stream);
+  if (mode != SSM_COMMIT_THRESHOLD && mode != SSM_COMMIT_TOPK && mode != SSM_COMMIT_MARGIN)
+    return SSM_ERR_INVALID_ARG;
+  if (block_len > 1024 || vocab > INT32_MAX) return SSM_ERR_UNSUPPORTED;
+  if (!logits || !masked || !conf || !argmax || !commit || !workspace) return SSM_ERR_INVALID_ARG;
+  if (mode == SSM_COMMIT_MARGIN && !p2) return SSM_ERR_INVALID_ARG;
+  if (topk < 0 || min_commit < 0 || !(threshold == threshold)) return SSM_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SSM_ERR_INVALID_ARG;
+  if (ws_bytes < ssm_unmask_workspace_size(batch, block_len, vocab, dtype)) return SSM_ERR_CAPACITY;
+  const int64_t rows = static_cast<int64_t>(batch) * block_len;
+  if (rows > 65535) return SSM_ERR_UNSUPPORTED;
+  // the top-k pass's own conditions, checked first so that an error enqueues nothing
+  const int esz = dtype == SSM_DTYPE_BF16 ? 2 : 4;
+  if (!ssm::aligned16(suffix_logits) || (vocab * esz) % 16 != 0) return SSM_ERR_UNSUPPORTED;
+  const int64_t nchunk = (vocab * esz + ssm::topk::kTopStageBytes - 1) / ssm::topk::kTopStageBytes;
+  if (ssm::topk::kTopStages * ssm::topk::kTopStageBytes + nchunk * ssm::topk::kTopThreads * esz + 128 >
+      ssm::topk::kTopMaxSmem)
+    return SSM_ERR_UNSUPPORTED;
+  // The two streaming passes back to back on the stream: the block rows' unmasking (its stream
+  // and commit kernels) and the suffix rows' top-k.  A single kernel serving both kinds of
+  // rows was measured slower than the two (it holds fewer bytes in flight per SM than the
+  // top-k pass alone), so the call enqueues the faster pair.
+  const ssm_status s = ssm_unmask(logits, dtype, batch, block_len, vocab, masked, mode, threshold, topk, min_commit,
+                                  conf, argmax, p2, commit, workspace, ws_bytes, stream);
+  if (s != SSM_OK) return s;
+  return ssm_suffix_topk(suffix_logits, dtype, n_suffix_rows, vocab, k, ids, probs, stream);
 }
 
 }  // extern "C"

@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
                                                   i32, vp, vp, vp, vp, vp]),
             "ssm_cache_append": (ctypes.c_int, [vp, vp, vp, i32, i32, i32, i32, f32, vp, vp, i64, i64, vp]),
             "ssm_suffix_topk": (ctypes.c_int, [vp, ctypes.c_int, i64, i64, i32, vp, vp, vp]),
+            "ssm_unmask_topk": (ctypes.c_int, [vp, ctypes.c_int, i32, i32, i64, vp, ctypes.c_int, f32, i32, i32,
+                                               vp, vp, vp, vp, vp, i64, i32, vp, vp, vp, sz, vp]),
             "ssm_early_stop": (ctypes.c_int, [vp, i32, i32, i32, i32, i32, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
@@ -103,7 +105,7 @@ def exported_symbols() -> Sequence[str]:
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
             "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
             "ssm_attention_varlen", "ssm_attention_varlen_rotate", "ssm_attention_varlen_core",
-            "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_noalloc",
+            "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_topk", "ssm_unmask_noalloc",
             "ssm_cache_append", "ssm_suffix_topk", "ssm_early_stop"]
 
 
@@ -344,6 +346,21 @@ def ssm_unmask(logits, masked, conf, argmax, commit, p2=None, mode: int = SSM_CO
         _ptr(logits), _dtype_code(logits), batch, block_len, vocab, _ptr(masked), mode, float(threshold), topk,
         min_commit, _ptr(conf), _ptr(argmax), _ptr(p2), _ptr(commit), _ptr(workspace), workspace.numel(),
         _stream(stream)))
+
+
+def ssm_unmask_topk(logits, masked, conf, argmax, commit, suffix_logits, k: int, ids, probs, p2=None,
+                    mode: int = SSM_COMMIT_THRESHOLD, threshold: float = 0.9, topk: int = 1, min_commit: int = 1,
+                    workspace=None, stream=None):
+    """ssm_unmask of the block rows and ssm_suffix_topk of suffix_logits [n_rows, vocab] in one pass."""
+    batch, block_len, vocab = logits.shape
+    n_suffix = suffix_logits.shape[0] if suffix_logits is not None else 0
+    need = ssm_unmask_workspace_size(batch, block_len, vocab, logits.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=logits.device)
+    _check("ssm_unmask_topk", lib().ssm_unmask_topk(
+        _ptr(logits), _dtype_code(logits), batch, block_len, vocab, _ptr(masked), mode, float(threshold), topk,
+        min_commit, _ptr(conf), _ptr(argmax), _ptr(p2), _ptr(commit), _ptr(suffix_logits), n_suffix, int(k),
+        _ptr(ids), _ptr(probs), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def ssm_unmask_noalloc(logits, masked, conf, argmax, commit, p2=None, mode: int = SSM_COMMIT_THRESHOLD,

@@ -4,9 +4,11 @@ Every mbarrier wait of the attention forward gives up after the library's wait l
 (ssm_set_wait_limit_ns), records SSM_ERR_TIMEOUT in the device error word and leaves its
 loop; the TMA producers then wait (under their own fixed 200 ms bound, not the shortened
 limit) for the copies they issued, the MMA warp for every MMA it issued, and the CTA frees
-its tensor memory before it exits.  With a 100 ns limit (also the try_wait suspend hint)
-nearly every wait that is not already complete at its first probe expires: the test checks
-the status and then that a launch at the default limit gives the same output as before.
+its tensor memory before it exits.  A limit below 20 us launches the forward's polling form
+(non-blocking probes, the limit checked between them), so with a 100 ns limit every wait
+that is not complete at its first probe within 100 ns expires -- the MMA warp's wait for
+the first P of a unit takes a softmax pass, about a microsecond.  The test checks the status
+and then that a launch at the default limit gives the same output as before.
 Nothing faults or hangs: the failure is a wait that runs out, read back by the host.
 """
 import pytest
