@@ -188,7 +188,10 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
       sn1[t] = s_sn[warp][8 * sub + 4 + t];
     }
     const int64_t row = gm.new_row + i;
-    if (p.row_prob && lane == 0) p.row_prob[row] = prob;
+    // a packed unit's softmax rows read their problem's key bounds from here in one load: the
+    // cache prefix length and the problem's new rows [new_row, new_row + n_new)
+    if (p.row_bounds && lane == 0)
+      p.row_bounds[row] = make_int4(gm.n_cache, static_cast<int>(gm.new_row), static_cast<int>(gm.new_row + gm.n_new), 0);
     for (int h0 = hoff; h0 < n_vec; h0 += 2 * HPP) {
       uint4 x1[2], x2[2];
 #pragma unroll
@@ -630,11 +633,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int lim = w.gm.n_cache, nlo = 0, nhi = w.gm.n_new;
       if (w.packed) {
         const bool mine = pr_u < w.urows;
-        const int b = p.row_prob[(w.orow0 + min(pr_u, w.urows - 1)) / p.grp];
-        const ssm_attn_problem q = p.problems[b];
-        lim = mine ? q.n_cache : lim;
-        nlo = mine ? static_cast<int>(q.new_row - w.gm.new_row) : nlo;
-        nhi = mine ? static_cast<int>(q.new_row - w.gm.new_row) + q.n_new : nhi;
+        const int4 bd = p.row_bounds[(w.orow0 + min(pr_u, w.urows - 1)) / p.grp];
+        lim = mine ? bd.x : lim;
+        nlo = mine ? bd.y - static_cast<int>(w.gm.new_row) : nlo;
+        nhi = mine ? bd.z - static_cast<int>(w.gm.new_row) : nhi;
       }
       for (int k = 0; k < jobs; ++k) {
         const int j = w.two ? k : 2 * k + x;
@@ -655,20 +657,28 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         const bool full_tile = __all_sync(0xffffffffu, full_row);
         // A row sees all keys of most sub-boxes or none of them (a whole sub-box of another
         // problem's new rows, or of cache rows past its prefix): the exponent's addend carries
-        // that (-inf: none), with no per-key work.  Only when some row of the warp sees part of
-        // a sub-box (one vote, warp-uniform) are the invalid keys set to -inf one by one; a row
-        // maximum (first tile of a unit, exact path) takes them all masked.
+        // that (-inf: none), with no per-key work.  Only in a sub-box that some row of the warp
+        // sees in part (votes, warp-uniform) are the invalid keys set to -inf one by one; a row
+        // maximum (first tile of a unit, exact path) takes every sub-box masked.
         bool whole = true;
 #pragma unroll
         for (int s4 = 0; s4 < 4; ++s4) whole = whole && ((lo[s4] == 0 && hi[s4] == kSub) || hi[s4] <= lo[s4]);
         const bool part_keys = !__all_sync(0xffffffffu, whole);
+        uint32_t an_bits = 0;
+#pragma unroll
+        for (int s4 = 0; s4 < 4; ++s4)
+          an_bits |= ((lo[s4] == 0 && hi[s4] == kSub) || hi[s4] <= lo[s4] ? 1u : 0u) << s4;
+        an_bits = __reduce_and_sync(0xffffffffu, an_bits);
         auto load_s = [&](bool for_max) {
           tmem_ld_x128(tS, sr);
           if (for_max ? !full_tile : part_keys) {
 #pragma unroll
-            for (int c = 0; c < kBN; ++c) {
-              const int cc = c & (kSub - 1);
-              sr[c] = (cc >= lo[c / kSub] && cc < hi[c / kSub]) ? sr[c] : __float_as_uint(-INFINITY);
+            for (int s4 = 0; s4 < 4; ++s4) {
+              if (!for_max && (an_bits & (1u << s4))) continue;
+#pragma unroll
+              for (int cc = 0; cc < kSub; ++cc)
+                sr[s4 * kSub + cc] =
+                    (cc >= lo[s4] && cc < hi[s4]) ? sr[s4 * kSub + cc] : __float_as_uint(-INFINITY);
             }
           }
         };
@@ -888,9 +898,9 @@ constexpr int kPartBoth = 0, kPartRotate = 1, kPartCore = 2;
 
 // Workspace of an attention call (byte offsets, each region 256-byte aligned): rotated
 // queries, rotated new keys, the unit plan of a ragged batch (header, then up to
-// max_pairs packed units) and the problem index of every new row.
+// max_pairs packed units) and, per new row, its problem's key bounds (16 bytes).
 struct WsLayout {
-  size_t khat, plan, row_prob, total;
+  size_t khat, plan, row_bounds, total;
   int max_pairs;
 };
 
@@ -900,8 +910,8 @@ WsLayout ws_layout(int64_t total_new, int32_t h_q, int32_t h_kv, int32_t d) {
   l.max_pairs = static_cast<int>((total_new * grp + 2 * kBM - 1) / (2 * kBM));
   l.khat = align_up(static_cast<size_t>(total_new) * h_q * d * 2, 256);
   l.plan = l.khat + align_up(static_cast<size_t>(total_new) * h_kv * d * 2, 256);
-  l.row_prob = l.plan + align_up(sizeof(AttnPlanHdr) + static_cast<size_t>(l.max_pairs) * sizeof(AttnPlanUnit), 256);
-  l.total = l.row_prob + align_up(static_cast<size_t>(total_new) * sizeof(int32_t), 256);
+  l.row_bounds = l.plan + align_up(sizeof(AttnPlanHdr) + static_cast<size_t>(l.max_pairs) * sizeof(AttnPlanUnit), 256);
+  l.total = l.row_bounds + align_up(static_cast<size_t>(total_new) * sizeof(int4), 256);
   return l;
 }
 
@@ -1001,7 +1011,7 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   const bool may_pack = !uniform && batch_or_np >= 2 &&
                         (cache_rows_per_b == 0 || 2 * static_cast<int64_t>(max_n_cache) > cache_rows_per_b);
   p.plan = may_pack ? reinterpret_cast<AttnPlanHdr*>(static_cast<uint8_t*>(workspace) + wl.plan) : nullptr;
-  p.row_prob = may_pack ? reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + wl.row_prob) : nullptr;
+  p.row_bounds = may_pack ? reinterpret_cast<int4*>(static_cast<uint8_t*>(workspace) + wl.row_bounds) : nullptr;
   p.scale_log2 = scale * kLog2e;
   p.out = static_cast<__nv_bfloat16*>(out);
   p.out_v8 = (reinterpret_cast<uintptr_t>(out) & 31u) == 0 ? 1 : 0;

@@ -58,7 +58,7 @@ struct AttnParams {
   int32_t new_rows_extent;           // row extent of the new-K/V maps (OOB coordinate)
   int32_t qrows_g;                   // ragged batches: rotated query rows of one kv head (head-major layout)
   AttnPlanHdr* plan;                 // ragged batches: the unit plan (header, then units), else null
-  int32_t* row_prob;                 // ragged batches: problem of each new row
+  int4* row_bounds;                  // ragged batches: per new row, its problem's (n_cache, new_row, new_row + n_new)
   int32_t units_per_pg;              // work units per (problem, kv head)
   int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)

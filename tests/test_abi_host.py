@@ -95,10 +95,10 @@ def test_workspace_sizes(lib):
     up = lambda x: (x + 255) // 256 * 256
     rows, pairs = 101 * 8, (101 * 8 + 255) // 256
     assert ssm.ssm_attention_workspace_size(rows, 32, 32, 128) == (
-        2 * rows * 32 * 128 * 2 + up(32 + 32 * pairs) + up(4 * rows))
+        2 * rows * 32 * 128 * 2 + up(32 + 32 * pairs) + up(16 * rows))
     rows, pairs = 8854, (8854 * 7 + 255) // 256    # GQA: 7 query heads per kv head pack 7 rows per query
     assert ssm.ssm_attention_workspace_size(rows, 28, 4, 128) == (
-        up(rows * 28 * 256) + up(rows * 4 * 256) + up(32 + 32 * pairs) + up(4 * rows))
+        up(rows * 28 * 256) + up(rows * 4 * 256) + up(32 + 32 * pairs) + up(16 * rows))
     # 126464 bf16 entries are 16 stages of 8192; segments aim at 912 work items per call
     ws = ssm.ssm_unmask_workspace_size(8, 32, 126464, torch.bfloat16)
     assert ws == 8 * 32 * 4 * 16   # 256 rows: four segments of four stages each, 16-byte partials
