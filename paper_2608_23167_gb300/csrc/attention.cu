@@ -156,6 +156,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
     const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max, int32_t n_prob,
     int32_t max_pairs, __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
+  pdl_enter();
   constexpr int LPH = D / 16;       // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
@@ -330,6 +331,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc128,
     const __grid_constant__ CUtensorMap tm_vc128, const __grid_constant__ CUtensorMap tm_kn128,
     const __grid_constant__ CUtensorMap tm_vn128, const AttnParams p) {
+  pdl_enter();
   using L = Layout<D>;
   constexpr int NP = L::NP;
   constexpr uint32_t kIdescQK = idesc_bf16_f32(kBM, kBN, false, false);
@@ -939,7 +941,8 @@ ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cud
       return SSM_ERR_CUDA;
     attr_set.fetch_or(bit);
   }
-  attn_fwd_kernel<D, PACKABLE, POLL><<<grid, kAttnThreads, L::ALLOC, st>>>(m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
+  ssm::launch_k(attn_fwd_kernel<D, PACKABLE, POLL>, dim3(grid), dim3(kAttnThreads), L::ALLOC, st,
+           m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
                                                                      m.kn128, m.vn128, p);
   return launch_status();
 }
@@ -1023,7 +1026,8 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     const int64_t items = static_cast<int64_t>(n_prob) * max_n_new;
     // persistent: three CTAs per SM at the kernel's register count
     const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, 3ll * num_sms()));
-    rope_pack_kernel<D><<<grid, kRopeWarps * 32, 0, st>>>(static_cast<const __nv_bfloat16*>(q),
+    ssm::launch_k(rope_pack_kernel<D>, dim3(grid), dim3(kRopeWarps * 32), 0, st,
+             static_cast<const __nv_bfloat16*>(q),
                                                           static_cast<const __nv_bfloat16*>(k_new), pos, p,
                                                           rope_theta, max_n_new, n_prob, wl.max_pairs, qhat,
                                                           khat);

@@ -62,6 +62,7 @@ __device__ __forceinline__ void zero_row(uint4* __restrict__ dst, int hvec) {
 }
 
 __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const BuildParams p) {
+  pdl_enter();
   __shared__ int32_t s_ids[kMaxK];
   __shared__ float s_w[kMaxK];
   __shared__ int32_t s_n;
@@ -247,7 +248,8 @@ ssm_status ssm_build_step_input(const int32_t* block_tokens, const int32_t* pref
   p.pos_out = pos_out;
   p.err = ssm::device_error_word();
   dim3 grid(rows, batch);
-  ssm::build_step_input_kernel<<<grid, ssm::kBuildThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+  ssm::launch_k(ssm::build_step_input_kernel, dim3(grid), dim3(ssm::kBuildThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+           p);
   return ssm::launch_status();
 }
 
@@ -285,7 +287,8 @@ ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t
   p.pos_out = pos_out;
   p.err = ssm::device_error_word();
   dim3 grid(max_rows, n_problems);
-  ssm::build_step_input_kernel<<<grid, ssm::kBuildThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+  ssm::launch_k(ssm::build_step_input_kernel, dim3(grid), dim3(ssm::kBuildThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+           p);
   return ssm::launch_status();
 }
 

@@ -28,6 +28,7 @@ __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
     const int32_t* __restrict__ pos, int32_t batch, int32_t n_rows, int32_t h_kv, float theta,
     __nv_bfloat16* __restrict__ k_cache, __nv_bfloat16* __restrict__ v_cache, int64_t cache_rows,
     int64_t start_row) {
+  pdl_enter();
   constexpr int LPH = D / 16;    // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;  // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
@@ -115,10 +116,12 @@ ssm_status ssm_cache_append(const void* k_new, const void* v_new, const int32_t*
   auto* kc = static_cast<__nv_bfloat16*>(k_cache);
   auto* vc = static_cast<__nv_bfloat16*>(v_cache);
   if (head_dim == 128)
-    ssm::cache_append_kernel<128><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, batch, n_rows, h_kv, rope_theta,
+    ssm::launch_k(ssm::cache_append_kernel<128>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st,
+             kn, vn, pos, batch, n_rows, h_kv, rope_theta,
                                                                          kc, vc, cache_rows, start_row);
   else
-    ssm::cache_append_kernel<64><<<grid, ssm::kAppendWarps * 32, 0, st>>>(kn, vn, pos, batch, n_rows, h_kv, rope_theta,
+    ssm::launch_k(ssm::cache_append_kernel<64>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st,
+             kn, vn, pos, batch, n_rows, h_kv, rope_theta,
                                                                         kc, vc, cache_rows, start_row);
   return ssm::launch_status();
 }

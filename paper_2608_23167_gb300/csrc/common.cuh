@@ -4,6 +4,7 @@
 
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <utility>
 
 #include "ssm.h"
 
@@ -35,5 +36,41 @@ inline ssm_status launch_status() {
 }
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Programmatic dependent launch.  Every libssm kernel launched directly on a stream carries
+// the programmatic stream serialization attribute and every kernel begins with pdl_enter():
+// griddepcontrol.wait blocks
+// until the grids it depends on have completed and their memory is visible (a kernel that
+// follows a non-libssm kernel or a copy waits for it as usual), then launch_dependents lets
+// the next kernel of the stream be scheduled while this one runs.  The next kernel's CTAs take
+// SM resources only as they free up and block in their own wait, so a dependent kernel's
+// launch latency and CTA start-up overlap this kernel's tail instead of following it.  Every
+// thread executes the wait before touching memory and before any return, so a kernel can
+// complete only after everything earlier on the stream has.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  // Direct launches only: replays of a captured CUDA graph already start each node right after
+  // its predecessor, and measured slower with programmatic edges, so launches being captured
+  // are ordinary ones (pdl_enter() is then a no-op wait)
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(st, &cap);
+  cfg.numAttrs = cap == cudaStreamCaptureStatusNone ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // errors: read by launch_status()
+}
 
 }  // namespace ssm

@@ -18,6 +18,7 @@ __global__ void __launch_bounds__(kEosThreads) early_stop_kernel(int32_t* __rest
                                                                  int32_t block_len, int32_t block_idx, int32_t eos_id,
                                                                  uint8_t* __restrict__ finished,
                                                                  int32_t* __restrict__ n_active) {
+  pdl_enter();
   __shared__ int s_first;
   const int64_t seq = blockIdx.x;
   if (finished[seq]) return;   // uniform over the CTA
@@ -51,7 +52,8 @@ extern "C" ssm_status ssm_early_stop(int32_t* tokens, int32_t batch, int32_t gen
   if (batch > INT32_MAX / 2) return SSM_ERR_UNSUPPORTED;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (n_active && cudaMemsetAsync(n_active, 0, sizeof(int32_t), st) != cudaSuccess) return SSM_ERR_CUDA;
-  ssm::early_stop_kernel<<<batch, ssm::kEosThreads, 0, st>>>(tokens, gen_len, block_len, block_idx, eos_id,
+  ssm::launch_k(ssm::early_stop_kernel, dim3(batch), dim3(ssm::kEosThreads), 0, st,
+           tokens, gen_len, block_len, block_idx, eos_id,
                                                              finished, n_active);
   return ssm::launch_status();
 }

@@ -112,6 +112,7 @@ struct SelectBatch {
 
 __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectBatch batch,
                                                              int32_t* __restrict__ positions) {
+  pdl_enter();
   __shared__ int32_t warp_tot[kSelThreads / 32];
   __shared__ int32_t base_s;
   const ssm_suffix_cfg cfg = batch.cfg[blockIdx.x];
@@ -180,7 +181,8 @@ ssm_status ssm_select_suffix_batch(const ssm_suffix_cfg* h_cfgs, int32_t n, int3
       sb.cfg[i] = h_cfgs[first + i];
       sb.offset[i] = off[first + i];
     }
-    ssm::select_kernel<<<cnt, ssm::kSelThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(sb, positions);
+    ssm::launch_k(ssm::select_kernel, dim3(cnt), dim3(ssm::kSelThreads), 0, reinterpret_cast<cudaStream_t>(stream),
+             sb, positions);
     const ssm_status ls = ssm::launch_status();
     if (ls != SSM_OK) return ls;
   }

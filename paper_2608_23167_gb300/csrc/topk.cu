@@ -64,6 +64,7 @@ template <typename T>
 __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restrict__ logits, int64_t vocab,
                                                               int64_t n_rows, int k, int32_t* __restrict__ ids,
                                                               float* __restrict__ probs) {
+  pdl_enter();
   constexpr int ESZ = sizeof(T);
   constexpr int EPV = 16 / ESZ;          // entries per 16-byte vector
   constexpr int EPW = EPV / 4;           // entries per word
@@ -252,11 +253,12 @@ ssm_status ssm_suffix_topk(const void* logits, ssm_dtype dtype, int64_t n_rows, 
   const int grid = static_cast<int>(std::min<int64_t>(n_rows, 5ll * ssm::num_sms()));
   if (dtype == SSM_DTYPE_BF16) {
     if (!ssm::topk_attr_set<ssm::topk_row_kernel<__nv_bfloat16>>()) return SSM_ERR_CUDA;
-    ssm::topk_row_kernel<__nv_bfloat16><<<grid, ssm::kTopThreads, smem, st>>>(
-        static_cast<const __nv_bfloat16*>(logits), vocab, n_rows, k, ids, probs);
+    ssm::launch_k(ssm::topk_row_kernel<__nv_bfloat16>, dim3(grid), dim3(ssm::kTopThreads), smem, st,
+             static_cast<const __nv_bfloat16*>(logits), vocab, n_rows, k, ids, probs);
   } else {
     if (!ssm::topk_attr_set<ssm::topk_row_kernel<float>>()) return SSM_ERR_CUDA;
-    ssm::topk_row_kernel<float><<<grid, ssm::kTopThreads, smem, st>>>(static_cast<const float*>(logits), vocab,
+    ssm::launch_k(ssm::topk_row_kernel<float>, dim3(grid), dim3(ssm::kTopThreads), smem, st,
+             static_cast<const float*>(logits), vocab,
                                                                      n_rows, k, ids, probs);
   }
   return ssm::launch_status();

@@ -135,6 +135,7 @@ template <typename T, bool NEED_SECOND>
 __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_stream_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
+  pdl_enter();
   constexpr int ESZ = sizeof(T);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
@@ -279,6 +280,7 @@ template <typename T>
 __global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_scalar_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t chunk, int n_chunks,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
+  pdl_enter();
   const int64_t row = blockIdx.y;
   if (!masked[row]) return;
   const int64_t c0 = static_cast<int64_t>(blockIdx.x) * chunk;
@@ -314,6 +316,7 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
     int block_len, int n_chunks, const uint8_t* __restrict__ masked, const Partial* __restrict__ part,
     int mode, float threshold, int topk, int min_commit, float* __restrict__ conf,
     int32_t* __restrict__ argmax, float* __restrict__ p2_out, uint8_t* __restrict__ commit) {
+  pdl_enter();
   extern __shared__ float smem[];
   float* s_conf = smem;                                               // [block_len]
   float* s_score = smem + block_len;                                  // [block_len]
@@ -468,14 +471,14 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
           !stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::unmask_stream_kernel<__nv_bfloat16, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
-        ssm::unmask_stream_kernel<__nv_bfloat16, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
     } else {
-      ssm::unmask_partial_scalar_kernel<__nv_bfloat16><<<grid, ssm::kUnmaskThreads, 0, st>>>(
-          x, vocab, plan.chunk, plan.n_chunks, masked, part);
+      ssm::launch_k(ssm::unmask_partial_scalar_kernel<__nv_bfloat16>, dim3(grid), dim3(ssm::kUnmaskThreads), 0, st,
+               x, vocab, plan.chunk, plan.n_chunks, masked, part);
     }
   } else {
     auto* x = static_cast<const float*>(logits);
@@ -484,21 +487,22 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
           !stream_attr_set<ssm::unmask_stream_kernel<float, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::unmask_stream_kernel<float, true><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
-        ssm::unmask_stream_kernel<float, false><<<stream_grid, ssm::kStreamThreads, stream_smem, st>>>(
-            x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+        ssm::launch_k(ssm::unmask_stream_kernel<float, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
     } else {
-      ssm::unmask_partial_scalar_kernel<float><<<grid, ssm::kUnmaskThreads, 0, st>>>(
-          x, vocab, plan.chunk, plan.n_chunks, masked, part);
+      ssm::launch_k(ssm::unmask_partial_scalar_kernel<float>, dim3(grid), dim3(ssm::kUnmaskThreads), 0, st,
+               x, vocab, plan.chunk, plan.n_chunks, masked, part);
     }
   }
   ssm_status s = ssm::launch_status();
   if (s != SSM_OK) return s;
   const int threads = ((block_len + 31) / 32) * 32;
   const size_t shm = static_cast<size_t>(block_len) * (2 * sizeof(float) + 2);
-  ssm::unmask_commit_kernel<<<batch, threads, shm, st>>>(block_len, plan.n_chunks, masked, part, mode,
+  ssm::launch_k(ssm::unmask_commit_kernel, dim3(batch), dim3(threads), shm, st,
+           block_len, plan.n_chunks, masked, part, mode,
                                                          threshold, topk, min_commit, conf, argmax, p2,
                                                          commit);
   return ssm::launch_status();
