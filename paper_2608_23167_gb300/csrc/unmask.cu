@@ -123,6 +123,17 @@ constexpr int kStageBytes = 16384;                     // one stage: 64 bytes pe
 constexpr int kStreamStages = 2;                       // chunks in flight per thread
 constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
 
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("min.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+
 // Running per-thread state over one segment: max m1 (first index idx), second
 // largest m2 (a repeated maximum counts twice) and s = sum exp(x - m1).
 struct RunState {
@@ -139,6 +150,8 @@ __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_st
   constexpr int ESZ = sizeof(T);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+  // NEED_SECOND: each thread's copy of its 64 bytes of the chunk that holds its running maximum
+  uint4* keep = reinterpret_cast<uint4*>(ring + kStreamStages * kStageBytes) + threadIdx.x * kVecPerThread;
   __shared__ Partial wpart[kStreamThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n_items = n_rows * n_seg;
@@ -213,17 +226,15 @@ __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_st
       }
       const float cm1 = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
       if constexpr (NEED_SECOND) {
-        // second largest of the running values after this chunk (a repeated maximum counts
-        // twice): only a chunk that raises the maximum needs its own second largest, which
-        // is rare once the row is under way
+        // Second largest (a repeated maximum counts twice) = the larger of the second largest
+        // inside the chunk that holds the maximum and the largest value of every other chunk.
+        // The second is kept as r.m2 per chunk; the first is taken once at the segment's end
+        // from a copy of the maximum's chunk (four 16-byte shared-memory stores whenever a
+        // chunk raises the maximum: on most chunks some lane of the warp does).
         if (cm1 > r.m1) {
-          float s2 = -INFINITY, m1l = -INFINITY;
+          r.m2 = fmaxf(r.m2, r.m1);
 #pragma unroll
-          for (int e = 0; e < PER; ++e) {
-            s2 = fmaxf(s2, fminf(m1l, f[e]));
-            m1l = fmaxf(m1l, f[e]);
-          }
-          r.m2 = fmaxf(fmaxf(r.m1, s2), r.m2);
+          for (int u = 0; u < kVecPerThread; ++u) keep[u] = v[u];
         } else {
           r.m2 = fmaxf(r.m2, cm1);
         }
@@ -259,6 +270,39 @@ __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_st
       if (cs.off >= cs.bytes) chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
     }
     // block partial of the segment: per-warp shuffles, then warp 0 merges the eight
+    if constexpr (NEED_SECOND) {
+      // the second largest inside the chunk that holds this thread's maximum
+      float s2 = -INFINITY;
+      if (r.m1 > -INFINITY) {
+        if constexpr (ESZ == 2) {
+          uint32_t mx = 0xFF80FF80u, sc = 0xFF80FF80u;
+#pragma unroll
+          for (int u = 0; u < kVecPerThread; ++u) {
+            const uint4 kv = keep[u];
+            const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              sc = bmax2(sc, bmin2(mx, w4[q]));
+              mx = bmax2(mx, w4[q]);
+            }
+          }
+          s2 = fmaxf(fminf(lo_bf16(mx), hi_bf16(mx)), fmaxf(lo_bf16(sc), hi_bf16(sc)));
+        } else {
+          float m1l = -INFINITY;
+#pragma unroll
+          for (int u = 0; u < kVecPerThread; ++u) {
+            const uint4 kv = keep[u];
+            const float w4[4] = {__uint_as_float(kv.x), __uint_as_float(kv.y), __uint_as_float(kv.z), __uint_as_float(kv.w)};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              s2 = fmaxf(s2, fminf(m1l, w4[q]));
+              m1l = fmaxf(m1l, w4[q]);
+            }
+          }
+        }
+      }
+      r.m2 = fmaxf(r.m2, s2);
+    }
     Partial pw{r.m1, r.s, r.idx, r.m2};
 #pragma unroll
     for (int d = 16; d >= 1; d >>= 1) pw = merge(pw, shfl_partial(pw, d));
@@ -459,7 +503,9 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));
-  const size_t stream_smem = ssm::kStreamStages * ssm::kStageBytes + 128;  // 96 KB: two CTAs per SM
+  // the ring (32 KB), plus with the second largest a 64-byte copy per thread (16 KB)
+  const size_t stream_smem = ssm::kStreamStages * ssm::kStageBytes + 128;
+  const size_t stream_smem2 = stream_smem + ssm::kStageBytes;
   const int64_t n_items = rows * plan.n_chunks;
   // one wave: three CTAs per SM are resident (registers), each takes ~2 items of ~kItemsTarget
   const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 3 * ssm::num_sms()));
@@ -467,11 +513,11 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
     if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem) ||
+      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem2) ||
           !stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem2, st,
                  x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
@@ -483,11 +529,11 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   } else {
     auto* x = static_cast<const float*>(logits);
     if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem) ||
+      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem2) ||
           !stream_attr_set<ssm::unmask_stream_kernel<float, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
+        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem2, st,
                  x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<float, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
