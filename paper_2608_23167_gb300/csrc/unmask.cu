@@ -141,16 +141,16 @@ struct RunState {
   int idx;
 };
 
-// (with the second largest tracked, the register cap keeps four CTAs per SM)
+// (three CTAs per SM: the grid is one wave of them)
 template <typename T, bool NEED_SECOND>
-__global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_stream_kernel(
+__global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
     const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
   pdl_enter();
   constexpr int ESZ = sizeof(T);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
-  // NEED_SECOND: each thread's copy of its 64 bytes of the chunk that holds its running maximum
+  // each thread's copy of its 64 bytes of the chunk that holds its running maximum
   uint4* keep = reinterpret_cast<uint4*>(ring + kStreamStages * kStageBytes) + threadIdx.x * kVecPerThread;
   __shared__ Partial wpart[kStreamThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -225,32 +225,21 @@ __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_st
         }
       }
       const float cm1 = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
-      if constexpr (NEED_SECOND) {
-        // Second largest (a repeated maximum counts twice) = the larger of the second largest
-        // inside the chunk that holds the maximum and the largest value of every other chunk.
-        // The second is kept as r.m2 per chunk; the first is taken once at the segment's end
-        // from a copy of the maximum's chunk (four 16-byte shared-memory stores whenever a
-        // chunk raises the maximum: on most chunks some lane of the warp does).
-        if (cm1 > r.m1) {
-          r.m2 = fmaxf(r.m2, r.m1);
-#pragma unroll
-          for (int u = 0; u < kVecPerThread; ++u) keep[u] = v[u];
-        } else {
-          r.m2 = fmaxf(r.m2, cm1);
-        }
-      }
+      // The argmax (first position of the maximum) and, when wanted, the second largest (a
+      // repeated maximum counts twice) are taken once, at the segment's end, from a copy of the
+      // maximum's chunk: a chunk that raises a lane's maximum only stores its 64 bytes (four
+      // 16-byte shared-memory stores; on most chunks some lane of the warp does).  The second
+      // largest is then the larger of the second largest inside that chunk and the largest
+      // value of every other chunk, which r.m2 keeps.
       if (cm1 > r.m1) {
+        if constexpr (NEED_SECOND) r.m2 = fmaxf(r.m2, r.m1);
+#pragma unroll
+        for (int u = 0; u < kVecPerThread; ++u) keep[u] = v[u];
+        r.idx = static_cast<int>(base);   // the kept chunk's first entry
         if (r.m1 > -INFINITY) r.s *= ex2((r.m1 - cm1) * kLog2e);
         r.m1 = cm1;
-        // first position of the new maximum among this thread's values (positions increase with e)
-        const int tbase = static_cast<int>(base) + static_cast<int>(threadIdx.x) * (16 / ESZ);
-        int best = INT_MAX;
-#pragma unroll
-        for (int e = PER - 1; e >= 0; --e) {
-          const int pos = tbase + (e / (16 / ESZ)) * kStreamThreads * (16 / ESZ) + (e % (16 / ESZ));
-          best = (f[e] == cm1) ? pos : best;
-        }
-        r.idx = best;
+      } else if constexpr (NEED_SECOND) {
+        r.m2 = fmaxf(r.m2, cm1);
       }
       if (r.m1 > -INFINITY) {
         const float mb = r.m1 * kLog2e;
@@ -270,38 +259,28 @@ __global__ void __launch_bounds__(kStreamThreads, NEED_SECOND ? 4 : 1) unmask_st
       if (cs.off >= cs.bytes) chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
     }
     // block partial of the segment: per-warp shuffles, then warp 0 merges the eight
-    if constexpr (NEED_SECOND) {
-      // the second largest inside the chunk that holds this thread's maximum
-      float s2 = -INFINITY;
-      if (r.m1 > -INFINITY) {
-        if constexpr (ESZ == 2) {
-          uint32_t mx = 0xFF80FF80u, sc = 0xFF80FF80u;
+    // the kept chunk: first position of the maximum and, when wanted, its second largest
+    if (r.m1 > -INFINITY) {
+      const int tbase = r.idx + static_cast<int>(threadIdx.x) * (16 / ESZ);
+      constexpr int EPV = 16 / ESZ;
+      int best = INT_MAX;
+      float s2 = -INFINITY, m1l = -INFINITY;
 #pragma unroll
-          for (int u = 0; u < kVecPerThread; ++u) {
-            const uint4 kv = keep[u];
-            const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
+      for (int u = kVecPerThread - 1; u >= 0; --u) {
+        const uint4 kv = keep[u];
+        const uint32_t w4[4] = {kv.x, kv.y, kv.z, kv.w};
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              sc = bmax2(sc, bmin2(mx, w4[q]));
-              mx = bmax2(mx, w4[q]);
-            }
-          }
-          s2 = fmaxf(fminf(lo_bf16(mx), hi_bf16(mx)), fmaxf(lo_bf16(sc), hi_bf16(sc)));
-        } else {
-          float m1l = -INFINITY;
-#pragma unroll
-          for (int u = 0; u < kVecPerThread; ++u) {
-            const uint4 kv = keep[u];
-            const float w4[4] = {__uint_as_float(kv.x), __uint_as_float(kv.y), __uint_as_float(kv.z), __uint_as_float(kv.w)};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              s2 = fmaxf(s2, fminf(m1l, w4[q]));
-              m1l = fmaxf(m1l, w4[q]);
-            }
+        for (int e = EPV - 1; e >= 0; --e) {
+          const float f = (ESZ == 2) ? ((e & 1) ? hi_bf16(w4[e >> 1]) : lo_bf16(w4[e >> 1])) : __uint_as_float(w4[e]);
+          best = (f == r.m1) ? tbase + u * kStreamThreads * EPV + e : best;
+          if constexpr (NEED_SECOND) {
+            s2 = fmaxf(s2, fminf(m1l, f));
+            m1l = fmaxf(m1l, f);
           }
         }
       }
-      r.m2 = fmaxf(r.m2, s2);
+      r.idx = best;
+      if constexpr (NEED_SECOND) r.m2 = fmaxf(r.m2, s2);
     }
     Partial pw{r.m1, r.s, r.idx, r.m2};
 #pragma unroll
@@ -503,9 +482,8 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));
-  // the ring (32 KB), plus with the second largest a 64-byte copy per thread (16 KB)
-  const size_t stream_smem = ssm::kStreamStages * ssm::kStageBytes + 128;
-  const size_t stream_smem2 = stream_smem + ssm::kStageBytes;
+  // the ring (32 KB) and a 64-byte copy per thread of its maximum's chunk (16 KB)
+  const size_t stream_smem = (ssm::kStreamStages + 1) * ssm::kStageBytes + 128;
   const int64_t n_items = rows * plan.n_chunks;
   // one wave: three CTAs per SM are resident (registers), each takes ~2 items of ~kItemsTarget
   const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 3 * ssm::num_sms()));
@@ -513,11 +491,11 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
     if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem2) ||
+      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem) ||
           !stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem2, st,
+        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
                  x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
@@ -529,11 +507,11 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   } else {
     auto* x = static_cast<const float*>(logits);
     if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem2) ||
+      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem) ||
           !stream_attr_set<ssm::unmask_stream_kernel<float, false>>(stream_smem))
         return SSM_ERR_CUDA;
       if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem2, st,
+        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
                  x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<float, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
