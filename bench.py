@@ -127,6 +127,7 @@ class StepInputs:
         self.step_tab = ssm.step_problems_tensor(
             [(i * w.block, i * n_prefix, int(self.suf_off[i]), int(self.row_off[i]), n_prefix, self.R[i],
               W.block_start(w, b)) for i, (_, b) in enumerate(self.problems)], device)
+        self.cfg_tab = ssm.suffix_cfgs_tensor(self.cfgs, device)
         self.attn_tab = ssm.attn_problems_tensor(
             [(int(self.row_off[i]), self.cache_row[i], self.rows[i], self.n_cache[i]) for i in range(n)], device)
         self.max_rows = max(self.rows)
@@ -187,12 +188,12 @@ class StepInputs:
         w = self.w
         if ev is not None:
             ev[0].record()
-        ssm.ssm_select_suffix_batch(self.positions, self.cfgs)
-        if ev is not None:
-            ev[1].record()
-        ssm.ssm_build_step_input_varlen(self.step_tab, self.n, self.max_rows, w.block, self.block_tokens,
-                                        self.positions, self.embed, self.mask_id, self.topk_ids, self.topk_prob,
-                                        w.topk, w.alpha, self.x, self.pos, prefix_tokens=self.prefix_tokens)
+            ev[1].record()   # selection is made inside the gather launch: its own stage is empty
+        # selection (Eqs. 1-5) and the sparse input (Eqs. 6-8) in one launch
+        ssm.ssm_select_build_step_input_varlen(self.step_tab, self.cfg_tab, self.n, self.max_rows, w.block,
+                                               self.block_tokens, self.embed, self.mask_id, self.topk_ids,
+                                               self.topk_prob, w.topk, w.alpha, self.x, self.pos, self.positions,
+                                               prefix_tokens=self.prefix_tokens)
         if ev is not None:
             ev[2].record()
         # the attention stage as its two launches (RoPE pre-pass, forward), timed apart
@@ -213,7 +214,7 @@ class StepInputs:
         if ev is not None:
             ev[5].record()
 
-    LAUNCHES_PER_STEP = 6   # select, build, rope_pack, attn_fwd, unmask stream, unmask commit
+    LAUNCHES_PER_STEP = 5   # select + build, rope_pack, attn_fwd, unmask stream, unmask commit
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -463,7 +464,8 @@ def stage_report(inp: "StepInputs", stage_ms, step_ms: float, peaks: dict) -> di
     gb = lambda nbytes, ms: nbytes / (ms * 1e-3) / 1e9 if ms > 0 else 0.0  # noqa: E731
     tf = lambda ms: flops / (ms * 1e-3) / 1e12 if ms > 0 else 0.0  # noqa: E731
     stages = {
-        "select_ms": sel_ms,
+        "select_ms": sel_ms, "select": "made inside the gather launch (ssm_select_build_step_input_varlen): "
+                                      "select_ms is an empty event pair, build_ms covers both",
         "build_ms": build_ms, "build_GBps": gb(inp.gather_bytes(), build_ms),
         "build_frac_hbm": gb(inp.gather_bytes(), build_ms) / hbm,
         "build_bytes": {"rows_read_distinct": inp.gather_rows_read(), "rows_read_gross": inp.gather_rows_read_gross(),

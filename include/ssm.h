@@ -182,6 +182,26 @@ ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t
                                        int32_t k, float alpha, void* x_out, int32_t* pos_out,
                                        ssm_stream_t stream);
 
+/* Selection and sparse input in one launch: ssm_select_suffix_batch followed by
+ * ssm_build_step_input_varlen, with every retained suffix row placing itself at
+ * the position of its rank in R_t (the closed form of Eqs. 2-5) instead of
+ * reading a selection written by an earlier launch.
+ *   cfgs            DEVICE array of n_problems ssm_suffix_cfg: problem p's
+ *                   selection; its |R_t| must equal problems[p].n_suffix
+ *                   (ssm_suffix_count), else SSM_ERR_DEVICE_INPUT is recorded
+ *                   and that problem's suffix rows are zeroed
+ *   suffix_pos_out  int32, R_t of problem p written at problems[p].suffix_off
+ *                   (the positions ssm_select_suffix_batch gives; may be NULL)
+ * Other arguments, outputs and errors as ssm_build_step_input_varlen, whose
+ * results this equals. */
+ssm_status ssm_select_build_step_input_varlen(const ssm_step_problem* problems, const ssm_suffix_cfg* cfgs,
+                                              int32_t n_problems, int32_t max_rows, int32_t block_len,
+                                              const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                              int32_t* suffix_pos_out, const void* embed, int64_t vocab,
+                                              int32_t hidden, int32_t mask_id, const int32_t* prev_topk_ids,
+                                              const float* prev_topk_prob, int32_t k, float alpha, void* x_out,
+                                              int32_t* pos_out, ssm_stream_t stream);
+
 /* ------------------------------------------------------------------------- */
 /* 3. Bidirectional attention over prefix cache + block + retained suffix     */
 /*    (Sec. 1 and Sec. 2: DLM attention is bidirectional; Sec. 3.2 "Sparse    */

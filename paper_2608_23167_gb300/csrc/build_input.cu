@@ -10,6 +10,7 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "suffix_geom.cuh"
 
 namespace ssm {
 namespace {
@@ -26,6 +27,8 @@ struct BuildParams {
   const int32_t* block_tokens;
   const int32_t* prefix_tokens;
   const int32_t* suffix_pos;
+  const ssm_suffix_cfg* cfgs;  // per problem: the selection, made here (suffix_pos unused), or null
+  int32_t* suffix_pos_out;     // with cfgs: R_t of every problem written here too (may be null)
   const uint4* embed;        // [vocab, hidden/8] 16-byte vectors
   int64_t vocab;
   int32_t hvec;              // hidden / 8
@@ -67,6 +70,7 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
   __shared__ float s_w[kMaxK];
   __shared__ int32_t s_n;
   __shared__ int32_t s_bad;
+  __shared__ int32_t s_mismatch;
 
   const int prob = blockIdx.y;
   const int r = blockIdx.x;
@@ -94,13 +98,15 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
   if (r >= rows) return;
   uint4* dst = p.x_out + (out_row + r) * p.hvec;
 
-  // original position id of this row (Sec. 3.2: retained tokens keep their positions)
-  if (threadIdx.x == 0 && p.pos_out && (p.problems || prob == 0)) {
+  // original position id of this row (Sec. 3.2: retained tokens keep their positions); with
+  // per-problem selections a retained suffix row's position is its rank in R_t mapped to the
+  // position in closed form (Eqs. 2-5, below), so no separate selection pass is needed
+  if (threadIdx.x == 0 && (p.problems || prob == 0) && !(p.cfgs && r >= n_prefix + p.block_len)) {
     int32_t pos;
     if (r < n_prefix) pos = r;
     else if (r < n_prefix + p.block_len) pos = block_start + (r - n_prefix);
     else pos = p.suffix_pos[suffix_off + (r - n_prefix - p.block_len)];
-    p.pos_out[(p.problems ? out_row : 0) + r] = pos;
+    if (p.pos_out) p.pos_out[(p.problems ? out_row : 0) + r] = pos;
   }
 
   if (r < n_prefix + p.block_len) {
@@ -119,6 +125,22 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
   const int64_t i = r - n_prefix - p.block_len;
   const int64_t cand = p.problems ? (suffix_off + i) * p.k
                                   : (static_cast<int64_t>(prob) * n_suffix + i) * p.k;
+  if (p.cfgs && threadIdx.x == 32) {
+    // this row's position, its rank i in R_t mapped in closed form, by a second warp while the
+    // first one gathers the candidates
+    const SuffixGeom g = make_geom(p.cfgs[prob]);
+    int32_t nl, nm, nt;
+    region_counts(g, nl, nm, nt);
+    if (nl + nm + nt != n_suffix) {   // the problem table disagrees with its selection
+      s_mismatch = 1;
+      record_error(p.err, SSM_ERR_DEVICE_INPUT);
+    } else {
+      s_mismatch = 0;
+      const int32_t pos = static_cast<int32_t>(retained_position(g, nl, nm, i));
+      if (p.pos_out) p.pos_out[out_row + r] = pos;
+      if (p.suffix_pos_out) p.suffix_pos_out[suffix_off + i] = pos;
+    }
+  }
   if (threadIdx.x == 0) {
     int n = 0, bad = 0;
     float z = 0.f;
@@ -141,7 +163,7 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
     if (bad) record_error(p.err, SSM_ERR_DEVICE_INPUT);
   }
   __syncthreads();
-  if (s_bad) {
+  if (s_bad || (p.cfgs && s_mismatch)) {
     zero_row(dst, p.hvec);
     return;
   }
@@ -289,6 +311,44 @@ ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t
   dim3 grid(max_rows, n_problems);
   ssm::launch_k(ssm::build_step_input_kernel, dim3(grid), dim3(ssm::kBuildThreads), 0, reinterpret_cast<cudaStream_t>(stream),
            p);
+  return ssm::launch_status();
+}
+
+ssm_status ssm_select_build_step_input_varlen(const ssm_step_problem* problems, const ssm_suffix_cfg* cfgs,
+                                              int32_t n_problems, int32_t max_rows, int32_t block_len,
+                                              const int32_t* block_tokens, const int32_t* prefix_tokens,
+                                              int32_t* suffix_pos_out, const void* embed, int64_t vocab,
+                                              int32_t hidden, int32_t mask_id, const int32_t* prev_topk_ids,
+                                              const float* prev_topk_prob, int32_t k, float alpha, void* x_out,
+                                              int32_t* pos_out, ssm_stream_t stream) {
+  ssm_status s = ssm::check_common(embed, vocab, hidden, mask_id, k, alpha, block_len, x_out);
+  if (s != SSM_OK) return s;
+  if (n_problems < 0 || max_rows < 0) return SSM_ERR_INVALID_ARG;
+  if (n_problems == 0 || max_rows == 0) return SSM_OK;
+  if (!problems || !cfgs || (block_len > 0 && !block_tokens)) return SSM_ERR_INVALID_ARG;
+  if (prev_topk_ids && k > 0 && !prev_topk_prob) return SSM_ERR_INVALID_ARG;
+  if (n_problems > 65535) return SSM_ERR_UNSUPPORTED;
+  ssm::BuildParams p{};
+  p.problems = problems;
+  p.n_problems = n_problems;
+  p.block_len = block_len;
+  p.block_tokens = block_tokens;
+  p.prefix_tokens = prefix_tokens;
+  p.cfgs = cfgs;
+  p.suffix_pos_out = suffix_pos_out;
+  p.embed = static_cast<const uint4*>(embed);
+  p.vocab = vocab;
+  p.hvec = hidden / 8;
+  p.mask_id = mask_id;
+  p.topk_ids = (k > 0) ? prev_topk_ids : nullptr;
+  p.topk_prob = prev_topk_prob;
+  p.k = k;
+  p.alpha = alpha;
+  p.x_out = static_cast<uint4*>(x_out);
+  p.pos_out = pos_out;
+  p.err = ssm::device_error_word();
+  ssm::launch_k(ssm::build_step_input_kernel, dim3(max_rows, n_problems), dim3(ssm::kBuildThreads), 0,
+                reinterpret_cast<cudaStream_t>(stream), p);
   return ssm::launch_status();
 }
 

@@ -8,88 +8,13 @@
 #include <vector>
 
 #include "common.cuh"
+#include "suffix_geom.cuh"
 
 namespace ssm {
 namespace {
 
-// Closed-form description of R_t for one configuration (shared by the host
-// count and the device membership test).
-struct SuffixGeom {
-  int64_t s0;          // first suffix position
-  int64_t end;         // one past the last generated position
-  int64_t tail_start;  // first position of the tail block
-  int64_t mid_first;   // start position of the first middle block
-  int32_t B, L, M, T;
-  int32_t n_sb;        // number of suffix blocks
-  int32_t nm;          // number of middle blocks
-  bool all_local;
-};
-
-__host__ __device__ inline SuffixGeom make_geom(const ssm_suffix_cfg& c) {
-  SuffixGeom g{};
-  const int32_t nb = c.gen_len / c.block_len;
-  g.B = c.block_len;
-  g.L = c.local_budget;
-  g.M = c.middle_budget;
-  g.T = c.tail_budget;
-  g.s0 = static_cast<int64_t>(c.prompt_len) + static_cast<int64_t>(c.block_idx + 1) * c.block_len;
-  g.end = static_cast<int64_t>(c.prompt_len) + c.gen_len;
-  g.n_sb = nb - 1 - c.block_idx;
-  g.tail_start = static_cast<int64_t>(c.prompt_len) + static_cast<int64_t>(nb - 1) * c.block_len;
-  g.all_local = static_cast<int64_t>(g.n_sb) * g.B <= g.L;
-  // middle blocks: suffix blocks other than the tail whose start is >= s0 + L
-  const int64_t first = (static_cast<int64_t>(g.L) + g.B - 1) / g.B;  // blocks touched by local
-  g.mid_first = g.s0 + first * g.B;
-  const int64_t nm = static_cast<int64_t>(g.n_sb) - 1 - first;
-  g.nm = nm > 0 ? static_cast<int32_t>(nm) : 0;
-  return g;
-}
-
-// Is tail-block offset `o` one of the T evenly spaced offsets (j*(B-1))/(T-1)?
-__host__ __device__ inline bool tail_keeps(const SuffixGeom& g, int64_t o) {
-  if (g.T <= 0) return false;
-  if (g.T >= g.B) return true;
-  if (g.T == 1) return o == 0;
-  const int64_t num = o * (g.T - 1);
-  const int64_t j = (num + (g.B - 2)) / (g.B - 1);  // smallest j with j*(B-1)/(T-1) >= o
-  return j <= g.T - 1 && (j * (g.B - 1)) / (g.T - 1) == o;
-}
-
-// Is middle block number `mi` (0-based among middle blocks) one of the kept ones?
-__host__ __device__ inline bool middle_keeps(const SuffixGeom& g, int64_t mi) {
-  if (g.nm <= g.M) return true;
-  if (g.M <= 0) return false;
-  const int64_t q = (mi * g.M + g.nm - 1) / g.nm;  // smallest q with q*nm/M >= mi
-  return q < g.M && (q * g.nm) / g.M == mi;
-}
-
-__host__ __device__ inline bool keeps(const SuffixGeom& g, int64_t pos) {
-  if (g.all_local) return true;
-  if (pos < g.s0 + g.L) return true;                               // Eq. 2
-  if (pos >= g.tail_start) return tail_keeps(g, pos - g.tail_start);  // Eq. 4
-  if (pos >= g.mid_first && (pos - g.mid_first) % g.B == 0)         // Eq. 3
-    return middle_keeps(g, (pos - g.mid_first) / g.B);
-  return false;
-}
-
 void host_counts(const ssm_suffix_cfg& c, int32_t* nl, int32_t* nmid, int32_t* nt) {
-  const SuffixGeom g = make_geom(c);
-  if (g.n_sb <= 0) {
-    *nl = *nmid = *nt = 0;
-    return;
-  }
-  if (g.all_local) {
-    *nl = g.n_sb * g.B;
-    *nmid = *nt = 0;
-    return;
-  }
-  *nl = g.L;
-  *nmid = std::min(g.nm, g.M);
-  // tail tokens not already local
-  int32_t t = 0;
-  for (int64_t o = 0; o < g.B; ++o)
-    if (g.tail_start + o >= g.s0 + g.L && tail_keeps(g, o)) ++t;
-  *nt = t;
+  region_counts(make_geom(c), *nl, *nmid, *nt);
 }
 
 ssm_status check_cfg(const ssm_suffix_cfg* c) {

@@ -72,6 +72,8 @@ def lib() -> ctypes.CDLL:
                                                     vp, vp, i32, f32, vp, vp, vp]),
             "ssm_build_step_input_varlen": (ctypes.c_int, [vp, i32, i32, i32, vp, vp, vp, vp, i64, i32, i32,
                                                            vp, vp, i32, f32, vp, vp, vp]),
+            "ssm_select_build_step_input_varlen": (ctypes.c_int, [vp, vp, i32, i32, i32, vp, vp, vp, vp, i64, i32,
+                                                                  i32, vp, vp, i32, f32, vp, vp, vp]),
             "ssm_attention_workspace_size": (sz, [i64, i32, i32, i32]),
             "ssm_attention": (ctypes.c_int, [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, f32, f32,
                                              vp, vp, vp, sz, vp]),
@@ -103,7 +105,7 @@ def lib() -> ctypes.CDLL:
 def exported_symbols() -> Sequence[str]:
     return ["ssm_status_str", "ssm_version", "ssm_get_device_error", "ssm_set_wait_limit_ns",
             "ssm_suffix_count", "ssm_select_suffix", "ssm_select_suffix_batch", "ssm_build_step_input",
-            "ssm_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
+            "ssm_build_step_input_varlen", "ssm_select_build_step_input_varlen", "ssm_attention_workspace_size", "ssm_attention",
             "ssm_attention_varlen", "ssm_attention_varlen_rotate", "ssm_attention_varlen_core",
             "ssm_unmask_workspace_size", "ssm_unmask", "ssm_unmask_topk", "ssm_unmask_noalloc",
             "ssm_cache_append", "ssm_suffix_topk", "ssm_early_stop"]
@@ -214,6 +216,22 @@ def step_problems_tensor(rows, device) -> torch.Tensor:
     for i, r in enumerate(rows):
         a[i] = tuple(r) + (0,)
     return torch.from_numpy(a.view(np.int64).copy()).to(device)
+
+
+def suffix_cfgs_tensor(cfgs, device) -> torch.Tensor:
+    """Packs (prompt, gen, block, block_idx, L, M, T) tuples into ssm_suffix_cfg records (28 bytes)."""
+    return torch.tensor([list(c) for c in cfgs], dtype=torch.int32).reshape(-1, 7).to(device)
+
+
+def ssm_select_build_step_input_varlen(problems, cfgs, n_problems: int, max_rows: int, block_len: int, block_tokens,
+                                       embed, mask_id: int, prev_topk_ids, prev_topk_prob, k: int, alpha: float,
+                                       x_out, pos_out=None, suffix_pos_out=None, prefix_tokens=None, stream=None):
+    """problems: device ssm_step_problem table; cfgs: device ssm_suffix_cfg table (suffix_cfgs_tensor)."""
+    vocab, hidden = embed.shape
+    _check("ssm_select_build_step_input_varlen", lib().ssm_select_build_step_input_varlen(
+        _ptr(problems), _ptr(cfgs), n_problems, max_rows, block_len, _ptr(block_tokens), _ptr(prefix_tokens),
+        _ptr(suffix_pos_out), _ptr(embed), vocab, hidden, mask_id, _ptr(prev_topk_ids), _ptr(prev_topk_prob), k,
+        float(alpha), _ptr(x_out), _ptr(pos_out), _stream(stream)))
 
 
 # ------------------------------------------------------------------------------ attention

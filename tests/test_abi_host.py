@@ -50,6 +50,25 @@ def test_suffix_count_matches_oracle(lib):
             assert ssm.ssm_suffix_count(P, G, B, b, L, M, T) == (nl, nm, nt)
 
 
+def test_suffix_count_closed_form_grid(lib):
+    """The region sizes in closed form (which the gather that selects as it builds also uses to
+    place every retained row) against the oracle's set construction over a grid of layouts:
+    budgets not multiples of the block, a local region reaching into the tail block, more middle
+    blocks than the middle budget, T = 0 / 1 / 2 / 3 / >= B."""
+    from paper_2608_23167_gb300 import ssm
+    n = 0
+    for B in (4, 8, 32):
+        for G in (B, 2 * B, 5 * B, 12 * B):
+            for L in (0, 1, B // 2, B, B + 3, 3 * B):
+                for M in (0, 1, 2, 5, 100):
+                    for T in (0, 1, 2, 3, B - 1, B, B + 2):
+                        for b in range(0, G // B, max(1, (G // B) // 4)):
+                            r, nl, nm, nt = O.select_suffix(7, G, B, b, L, M, T)
+                            assert ssm.ssm_suffix_count(7, G, B, b, L, M, T) == (nl, nm, nt), (G, B, b, L, M, T)
+                            n += 1
+    assert n > 2000
+
+
 def test_argument_validation_without_device(lib):
     from paper_2608_23167_gb300 import ssm
     cfg = ssm.SuffixCfg(0, 100, 32, 0, 32, 8, 4)          # G % B != 0
