@@ -82,6 +82,7 @@ struct Layout {
 // ---------------------------------------------------------------------------
 
 constexpr int kRopeWarps = 8;
+constexpr int kRopePasses = 4;  // head passes of a warp in flight (a lane's loads: 2 x this, 16 bytes each)
 
 // Problem whose new rows contain row r: the last problem starting at or before r
 // (problems of a packable plan start at increasing rows).
@@ -149,10 +150,10 @@ __device__ void attn_plan_warp(const AttnParams& p, int n_prob, int64_t total_ne
 // + row (items past a problem's row count are skipped).  A row's D/2 angles are
 // formed once (two per lane) and shared through shared memory; a lane then owns
 // eight rotation pairs (i, i + D/2) of one head vector (D/16 lanes per head,
-// 16-byte loads and stores, two head passes in flight).  The rotation is
+// 16-byte loads and stores, kRopePasses head passes in flight).  The rotation is
 // rope.cuh's (inverse frequencies once per CTA).
 template <int D>
-__global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
+__global__ void __launch_bounds__(kRopeWarps * 32, 3) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
     const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max, int32_t n_prob,
     int32_t max_pairs, __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
@@ -193,10 +194,10 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
     // cache prefix length and the problem's new rows [new_row, new_row + n_new)
     if (p.row_bounds && lane == 0)
       p.row_bounds[row] = make_int4(gm.n_cache, static_cast<int>(gm.new_row), static_cast<int>(gm.new_row + gm.n_new), 0);
-    for (int h0 = hoff; h0 < n_vec; h0 += 2 * HPP) {
-      uint4 x1[2], x2[2];
+    for (int h0 = hoff; h0 < n_vec; h0 += kRopePasses * HPP) {
+      uint4 x1[kRopePasses], x2[kRopePasses];
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
+      for (int u = 0; u < kRopePasses; ++u) {
         const int h = h0 + u * HPP;
         if (h < n_vec) {
           const __nv_bfloat16* src = h < p.h_q ? q + (row * p.h_q + h) * D : k + (row * p.h_kv + (h - p.h_q)) * D;
@@ -205,7 +206,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32) rope_pack_kernel(
         }
       }
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
+      for (int u = 0; u < kRopePasses; ++u) {
         const int h = h0 + u * HPP;
         if (h >= n_vec) continue;
         uint2 ya, yb, yc, yd;
@@ -642,11 +643,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       }
       for (int k = 0; k < jobs; ++k) {
         const int j = w.two ? k : 2 * k + x;
-        ok = warp_wait<POLL>(&bars[S_FULL + x], sj & 1, p.wait_ns);
-        if (!ok) break;
-        tc_fence_after_sync();
-        uint32_t sr[kBN];
-        // valid keys of each 32-key sub-box of the tile for this row: columns [lo, hi)
+        // The tile's masking plan is made while the tensor core still computes S (it depends
+        // only on the tile index and the row's bounds): valid keys of each 32-key sub-box of
+        // the tile for this row, columns [lo, hi)
         int lo[4], hi[4];
         bool full_row;
         if (w.packed) {
@@ -671,6 +670,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         for (int s4 = 0; s4 < 4; ++s4)
           an_bits |= ((lo[s4] == 0 && hi[s4] == kSub) || hi[s4] <= lo[s4] ? 1u : 0u) << s4;
         an_bits = __reduce_and_sync(0xffffffffu, an_bits);
+        ok = warp_wait<POLL>(&bars[S_FULL + x], sj & 1, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after_sync();
+        uint32_t sr[kBN];
         auto load_s = [&](bool for_max) {
           tmem_ld_x128(tS, sr);
           if (for_max ? !full_tile : part_keys) {
@@ -1024,8 +1027,10 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   const int n_prob = batch_or_np;
   if (part != kPartCore) {
     const int64_t items = static_cast<int64_t>(n_prob) * max_n_new;
-    // persistent: three CTAs per SM at the kernel's register count
-    const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, 3ll * num_sms()));
+    // persistent: as many CTAs per SM as fit (three at the kernel's register bound)
+    static const int per_sm = resident_ctas(rope_pack_kernel<D>, kRopeWarps * 32, 0);
+    const int grid = static_cast<int>(
+        std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, static_cast<int64_t>(per_sm) * num_sms()));
     ssm::launch_k(rope_pack_kernel<D>, dim3(grid), dim3(kRopeWarps * 32), 0, st,
              static_cast<const __nv_bfloat16*>(q),
                                                           static_cast<const __nv_bfloat16*>(k_new), pos, p,

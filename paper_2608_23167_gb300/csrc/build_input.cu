@@ -56,8 +56,19 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
+// A row copy with every thread's loads issued before its stores (four 16-byte vectors per
+// thread in flight, not one load-store round trip per vector).
 __device__ __forceinline__ void copy_row(const uint4* __restrict__ src, uint4* __restrict__ dst, int hvec) {
-  for (int v = threadIdx.x; v < hvec; v += kBuildThreads) dst[v] = __ldg(src + v);
+  constexpr int U = 4;
+  for (int v0 = threadIdx.x; v0 < hvec; v0 += U * kBuildThreads) {
+    uint4 t[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (v0 + u * kBuildThreads < hvec) t[u] = __ldg(src + v0 + u * kBuildThreads);
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (v0 + u * kBuildThreads < hvec) dst[v0 + u * kBuildThreads] = t[u];
+  }
 }
 
 __device__ __forceinline__ void zero_row(uint4* __restrict__ dst, int hvec) {
@@ -141,26 +152,35 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
       if (p.suffix_pos_out) p.suffix_pos_out[suffix_off + i] = pos;
     }
   }
-  if (threadIdx.x == 0) {
-    int n = 0, bad = 0;
+  if (threadIdx.x < 32) {
+    // the k candidates (id, p) of the previous step, lane j loading candidate j (k <= 32), so
+    // that their loads are in flight together; an id of -1 is absent, an id outside the
+    // vocabulary is an input error
+    const int lane = threadIdx.x;
+    const bool have = p.topk_ids != nullptr && lane < p.k;
+    const int32_t id = have ? p.topk_ids[cand + lane] : -1;
+    const float pj = have ? p.topk_prob[cand + lane] : 0.f;
+    const bool bad = id != -1 && (id < 0 || id >= p.vocab);
+    const unsigned use = __ballot_sync(0xffffffffu, id != -1 && !bad);
+    const unsigned badm = __ballot_sync(0xffffffffu, bad);
+    // the renormaliser sum(p) over the kept candidates, added in candidate order
     float z = 0.f;
-    if (p.topk_ids) {
-      for (int j = 0; j < p.k; ++j) {
-        const int32_t id = p.topk_ids[cand + j];
-        if (id == -1) continue;
-        if (id < 0 || id >= p.vocab) { bad = 1; continue; }
-        s_ids[n] = id;
-        s_w[n] = p.topk_prob[cand + j];
-        z += s_w[n];
-        ++n;
-      }
+    for (int j = 0; j < p.k; ++j) {
+      const float w = __shfl_sync(0xffffffffu, pj, j);
+      if ((use >> j) & 1u) z += w;
     }
-    if (!(z > 0.f)) n = 0;                       // no prediction: the row keeps e_mask
+    const int n = (z > 0.f) ? __popc(use) : 0;   // no prediction: the row keeps e_mask
     const float scale = n ? p.alpha / z : 0.f;   // alpha * p_j / sum(p) = alpha * p~_j
-    for (int j = 0; j < n; ++j) s_w[j] *= scale;
-    s_n = n;
-    s_bad = bad;
-    if (bad) record_error(p.err, SSM_ERR_DEVICE_INPUT);
+    if (n && ((use >> lane) & 1u)) {
+      const int slot = __popc(use & ((1u << lane) - 1u));
+      s_ids[slot] = id;
+      s_w[slot] = pj * scale;
+    }
+    if (lane == 0) {
+      s_n = n;
+      s_bad = badm != 0u;
+      if (badm) record_error(p.err, SSM_ERR_DEVICE_INPUT);
+    }
   }
   __syncthreads();
   if (s_bad || (p.cfgs && s_mismatch)) {
@@ -177,32 +197,30 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
   for (int v = threadIdx.x; v < p.hvec; v += kBuildThreads) {
     float acc[8];
     {
-      float m[8];
-      unpack8(__ldg(e_mask + v), m);
+      const uint4 mv = __ldg(e_mask + v);
 #pragma unroll
       for (int c = 0; c < 8; ++c) acc[c] = 0.f;
-      // gather the candidate rows four at a time so several loads are in flight
-      int j = 0;
-      for (; j + 4 <= n; j += 4) {
-        uint4 e4[4];
+      // gather the candidate rows six at a time: all of a chunk's loads (and the [MASK]
+      // row's) are in flight together; the products are added in candidate order
+      constexpr int C = 6;
+      for (int j = 0; j < n; j += C) {
+        uint4 ev[C];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) e4[u] = __ldg(p.embed + static_cast<int64_t>(s_ids[j + u]) * p.hvec + v);
+        for (int u = 0; u < C; ++u)
+          if (j + u < n) ev[u] = __ldg(p.embed + static_cast<int64_t>(s_ids[j + u]) * p.hvec + v);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          float f[8];
-          unpack8(e4[u], f);
-          const float w = s_w[j + u];
+        for (int u = 0; u < C; ++u) {
+          if (j + u < n) {
+            float f[8];
+            unpack8(ev[u], f);
+            const float w = s_w[j + u];
 #pragma unroll
-          for (int c = 0; c < 8; ++c) acc[c] = fmaf(w, f[c], acc[c]);
+            for (int c = 0; c < 8; ++c) acc[c] = fmaf(w, f[c], acc[c]);
+          }
         }
       }
-      for (; j < n; ++j) {
-        float f[8];
-        unpack8(__ldg(p.embed + static_cast<int64_t>(s_ids[j]) * p.hvec + v), f);
-        const float w = s_w[j];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) acc[c] = fmaf(w, f[c], acc[c]);
-      }
+      float m[8];
+      unpack8(mv, m);
 #pragma unroll
       for (int c = 0; c < 8; ++c) acc[c] = fmaf(keep, m[c], acc[c]);
     }

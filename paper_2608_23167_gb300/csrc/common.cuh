@@ -30,6 +30,15 @@ inline int num_sms() {
   return n;
 }
 
+// CTAs of `kernel` that fit on one SM at `threads` threads and `smem` bytes of dynamic shared
+// memory (at least 1): the grid size of a persistent kernel is this times the SM count.
+template <typename Kernel>
+inline int resident_ctas(Kernel kernel, int threads, size_t smem) {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, smem) != cudaSuccess || n < 1) return 1;
+  return n;
+}
+
 inline ssm_status launch_status() {
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SSM_OK : SSM_ERR_CUDA;
