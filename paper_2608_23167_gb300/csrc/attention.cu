@@ -507,12 +507,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           int& pv = x ? pv1 : pv0;
           if (!wait_o_free(x)) return false;
           // the K/V watcher's share of this phase vouches for V(jp) and this slot's next K tile
-          if (!warp_wait<POLL>(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
           const int vi = vbase + jp;
-          tc_fence_after_sync();
           const uint64_t vb = dV + static_cast<uint64_t>(((vi % kVStages) * L::TILE) >> 4);
           const uint32_t d_tmem = tmem + kOCol + x * D, a_tmem = tmem + x * kBN;
           const uint32_t acc0 = k > 0 ? 1u : 0u;
+          if (!warp_wait<POLL>(&bars[P_FULL + x], pv & 1, p.wait_ns)) return false;
+          tc_fence_after_sync();
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk)
             umma_bf16_ts_if(leader, d_tmem, a_tmem + kk * 8, vb + static_cast<uint64_t>((kk * 16 * 128) >> 4),
@@ -527,15 +527,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           const int x = t & 1;
           const int j = w.two ? (t >> 1) : t;
           const int ki = kbase + j;
-          if ((x ? kx1 : kx0) > 0)
-            ok = issue_pv(x);  // the watcher's share of P_FULL vouches for this slot's next K tile too
-          else
-            ok = warp_wait<POLL>(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
-          if (!ok) break;
-          tc_fence_after_sync();
           const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
           const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
           const uint32_t s_tmem = tmem + x * kBN;
+          if ((x ? kx1 : kx0) > 0) {
+            // the watcher's share of P_FULL vouches for this slot's next K tile too; issue_pv's
+            // fence after that wait orders this QK^T as well
+            ok = issue_pv(x);
+          } else {
+            ok = warp_wait<POLL>(&bars[K_FULL + ki % kKStages], (ki / kKStages) & 1, p.wait_ns);
+            if (ok) tc_fence_after_sync();
+          }
+          if (!ok) break;
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint64_t off = static_cast<uint64_t>(((kk >> 2) * kPanel + (kk & 3) * 32) >> 4);
