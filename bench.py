@@ -380,31 +380,56 @@ def time_stages(inp: StepInputs, reps: int, flush) -> np.ndarray:
     return a.mean(axis=0)
 
 
-def time_e2e(inp: StepInputs, steps: int, warmup: int, dist_on: bool):
-    """The same step through the public API with host buffers: per step, the step's
-    inputs are copied from pinned host memory and the decode result is read back."""
-    ins = [inp.block_tokens, inp.topk_ids, inp.topk_prob, inp.q, inp.k, inp.v, inp.logits]
-    host_in = [t.cpu().pin_memory() for t in ins]
-    outs = [inp.commit, inp.argmax, inp.conf]
-    host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
-    h2d = sum(t.numel() * t.element_size() for t in host_in)
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
+def time_e2e(bufs, steps: int, warmup: int, dist_on: bool):
+    """The same step through the public API with host buffers: per step, the step's inputs are
+    copied from pinned host memory and the decode result (commit, argmax, conf) is read back.
 
-    def one():
-        for d, h in zip(ins, host_in):
-            d.copy_(h, non_blocking=True)
-        inp.step()
-        for h, d in zip(host_out, outs):
+    With two input sets (`bufs`, each a StepInputs of the same workload) the copies of step
+    i + 1 run on a copy stream while step i computes on the current stream (double buffering:
+    a buffer is refilled only after the step that read it has finished); with one, copy and
+    compute alternate on one stream.  Returns (ms for `steps` steps, bytes in, bytes out per step)."""
+    def ins(b):
+        return [b.block_tokens, b.topk_ids, b.topk_prob, b.q, b.k, b.v, b.logits]
+
+    def outs(b):
+        return [b.commit, b.argmax, b.conf]
+
+    host_in = [t.cpu().pin_memory() for t in ins(bufs[0])]
+    host_out = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs(b)] for b in bufs]
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out[0])
+    compute = torch.cuda.current_stream()
+    copy = torch.cuda.Stream() if len(bufs) > 1 else compute
+    done = [torch.cuda.Event() for _ in bufs]     # the step that read buffer b has finished
+    loaded = [torch.cuda.Event() for _ in bufs]   # buffer b holds the next step's inputs
+    for e in done:
+        e.record(compute)
+
+    def one(i):
+        k = i % len(bufs)
+        b = bufs[k]
+        with torch.cuda.stream(copy):
+            copy.wait_event(done[k])
+            for d, h in zip(ins(b), host_in):
+                d.copy_(h, non_blocking=True)
+            loaded[k].record(copy)
+        compute.wait_event(loaded[k])
+        b.step()
+        # the step has read its inputs: the buffer may be refilled (its outputs, read back below,
+        # are rewritten only by a later step on this stream); recorded ahead of the read-back,
+        # which otherwise queues behind the next copy in and stalls the pipeline
+        done[k].record(compute)
+        for h, d in zip(host_out[k], outs(b)):
             h.copy_(d, non_blocking=True)
 
-    for _ in range(warmup):
-        one()
+    for i in range(warmup):
+        one(i)
     torch.cuda.synchronize()
     if dist_on:
         torch.distributed.barrier()
     t0 = time.perf_counter()
-    for _ in range(steps):
-        one()
+    for i in range(steps):
+        one(i)
     torch.cuda.synchronize()
     if dist_on:
         torch.distributed.barrier()
@@ -832,10 +857,18 @@ def main():
 
     e2e = None
     if not args.no_e2e:
-        e_ms, h2d, d2h = time_e2e(inp, args.steps, min(args.warmup, 5), dist_on)
+        # a second input set for double buffering (the embedding table, cache and workspaces are
+        # per set too: about 3 GB for the long sweep)
+        inp2 = StepInputs(w, dev)
+        e_ms, h2d, d2h = time_e2e([inp, inp2], args.steps, min(args.warmup, 5), dist_on)
+        del inp2
+        torch.cuda.empty_cache()
         e_ms = reduce_max(e_ms, dev, dist_on)
         e2e = {"value": inp.n * args.steps * world / (e_ms / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "how": "host clock over the steps; per step its inputs copied from pinned host memory (on a copy "
+                      "stream, into one of two input sets, while the previous step computes) and commit, argmax "
+                      "and conf read back"}
 
     peaks, peak_src = load_peaks()
     rep = stage_report(inp, stage_ms, total_ms / args.steps, peaks)
