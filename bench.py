@@ -17,6 +17,7 @@ are independent replicas: the path has no exchange step.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import math
 import os
@@ -65,7 +66,11 @@ class StepInputs:
         self.n = n
         self.cfgs = [(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail) for _, b in self.problems]
         self.R = [suffix_positions(w, b) for _, b in self.problems]
-        n_prefix = 0 if w.prefix_cached else w.prompt
+        # without a prefix cache the step recomputes the prompt and the blocks already decoded
+        # (one block index per batch here, so one prefix length)
+        if not w.prefix_cached and len(set(blocks)) != 1:
+            raise ValueError("a workload without prefix cache takes one block index per step")
+        n_prefix = 0 if w.prefix_cached else w.prompt + blocks[0] * w.block
         self.n_prefix = n_prefix
         self.rows = [n_prefix + w.block + r for r in self.R]          # sparse-input rows per problem
         self.row_off = np.concatenate([[0], np.cumsum(self.rows)]).astype(np.int64)
@@ -84,8 +89,10 @@ class StepInputs:
                 self.cache_rows = w.prompt + w.gen
                 self.cache_row = [0 for _ in self.problems]
             else:
-                self.cache_rows = w.batch * w.prompt
-                self.cache_row = [s * w.prompt for s, _ in self.problems]
+                # one cache per sequence, long enough for its largest block index's prefix
+                seg = w.prompt + max(blocks) * w.block
+                self.cache_rows = w.batch * seg
+                self.cache_row = [s * seg for s, _ in self.problems]
             self.n_cache = [w.prompt + b * w.block for _, b in self.problems]
             self.k_cache = torch.randn((self.cache_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
             self.v_cache = torch.randn((self.cache_rows, w.h_kv, w.head_dim), generator=g, device=device).to(torch.bfloat16)
@@ -287,7 +294,8 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": n}
 
 
-def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool, use_graph: bool = True):
+def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool, use_graph: bool = True,
+               stages: bool = True):
     """Times K steps.  The step (its five launches) is captured once in a CUDA graph and
     replayed, so the device time is not paced by the host's per-call work.  When a step
     reads less than twice the L2, the L2 is flushed before every timed step, outside that
@@ -332,7 +340,7 @@ def time_steps(inp: StepInputs, steps: int, warmup: int, dist_on: bool, use_grap
         total_ms = sum(a.elapsed_time(b) for a, b in evs)
     if dist_on:
         torch.distributed.barrier()
-    stage_ms = time_stages(inp, min(steps, 50), flush)
+    stage_ms = time_stages(inp, min(steps, 50), flush) if stages else None
     desc = {"launch": "CUDA graph of the step, replayed" if use_graph else "eager calls",
             "l2": ("inputs larger than L2 (each step reads ~%.0f MB)" % (inp.step_bytes() / 1e6)) if flush is None
             else ("L2 flushed before each timed step (%d MB written outside the step's events; each step reads "
@@ -473,8 +481,8 @@ def oracle_sample(w: W.Workload, budget_s: float, seed: int = 99):
             step //= 2
         order = spread
     done, t_used, used = 0, 0.0, []
-    n_prefix = 0 if w.prefix_cached else w.prompt
     for b in order * max(1, w.batch):
+        n_prefix = 0 if w.prefix_cached else w.prompt + b * w.block
         r, *_ = O.select_suffix(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
         R = len(r)
         n_new = n_prefix + w.block + R
@@ -585,7 +593,7 @@ def time_eager(inp: "StepInputs", steps: int, warmup: int) -> float:
     return total / steps
 
 
-def measure_configs(dev, steps: int, warmup: int, peaks: dict, skip: str) -> dict:
+def measure_configs(dev, steps: int, warmup: int, peaks: dict, skip: str, sweep_steps: int = 10) -> dict:
     """The other workloads, one bench step each as graph replays and as eager calls: denoising
     steps/s, the step-floor fraction, attention TFLOP/s against the burst peak, gather and unmask
     GB/s against the measured copy bandwidth."""
@@ -619,7 +627,31 @@ def measure_configs(dev, steps: int, warmup: int, peaks: dict, skip: str) -> dic
         }
         del inp
         torch.cuda.empty_cache()
+        out[name]["sweep"] = time_sweep(w, dev, sweep_steps, warmup)
     return out
+
+
+def time_sweep(w: W.Workload, dev, steps: int, warmup: int) -> dict:
+    """Every block index of the generation, one bench step each (the workload's batch at that
+    index), as graph replays behind an L2 flush: the denoising steps of a whole generation
+    pass.  Block 0 has the longest suffix; later blocks have shorter suffixes and longer
+    prefixes (a longer cache, or without a cache a longer recomputed prefix)."""
+    from paper_2608_23167_gb300 import ssm
+    per_b = []
+    for b in range(w.n_blocks):
+        inp = StepInputs(dataclasses.replace(w, block_indices=(b,)), dev)
+        total_ms, _, _ = time_steps(inp, steps, warmup, False, use_graph=True, stages=False)
+        if ssm.ssm_get_device_error() != 0:
+            raise RuntimeError(f"device error in the {w.name} sweep at block {b}")
+        per_b.append(total_ms / steps)
+        del inp
+        torch.cuda.empty_cache()
+    tot = sum(per_b)
+    return {"blocks": w.n_blocks, "timed_steps_per_block": steps, "ms_per_step_mean": tot / len(per_b),
+            "ms_per_step_min": min(per_b), "ms_per_step_max": max(per_b),
+            "value": w.batch * len(per_b) / (tot * 1e-3), "unit": UNIT,
+            "how": "one graph-replayed step per block index 0..n_blocks-1 (the workload's batch at that index), "
+                   "L2 flushed before each; value = denoising steps of the sweep / summed step times"}
 
 
 def oracle_one_thread(w: W.Workload, budget_s: float) -> dict:
