@@ -351,12 +351,12 @@ ssm_status ssm_unmask_topk(const void* logits, ssm_dtype dtype, int32_t batch, i
  * program whose device memory is owned by another framework's allocator, or a
  * code path where allocation is not permitted.  This entry point takes the
  * same arguments as ssm_unmask minus the workspace and allocates nothing: its
- * scratch is a fixed 1 MiB array in device global memory that the library
+ * scratch is a fixed 2 MiB array in device global memory that the library
  * holds on every GPU that loads it, until the process exits.
  *   - Limit: ssm_unmask_workspace_size(batch, block_len, vocab, dtype) must be
- *     at most 1 MiB (with a 126464-entry bf16 vocabulary that holds every
- *     call of up to 65535 positions, the most ssm_unmask takes); larger calls
- *     return SSM_ERR_CAPACITY and enqueue nothing.
+ *     at most 2 MiB (with a 126464-entry bf16 or fp32 vocabulary that holds
+ *     every call of up to 65535 positions, the most ssm_unmask takes); larger
+ *     calls return SSM_ERR_CAPACITY and enqueue nothing.
  *   - The first call on a device looks up the array's device address (with
  *     that device current); make that first call before any stream capture.
  *     The address is kept for the life of the process: a cudaDeviceReset makes

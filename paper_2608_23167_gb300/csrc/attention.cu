@@ -146,37 +146,60 @@ __device__ void attn_plan_warp(const AttnParams& p, int n_prob, int64_t total_ne
   }
 }
 
-// Persistent warps over (problem, row) items, item = problem * rows_per_problem_max
-// + row (items past a problem's row count are skipped).  A row's D/2 angles are
-// formed once (two per lane) and shared through shared memory; a lane then owns
-// eight rotation pairs (i, i + D/2) of one head vector (D/16 lanes per head,
-// 16-byte loads and stores, kRopePasses head passes in flight).  The rotation is
-// rope.cuh's (inverse frequencies once per CTA).
+// Persistent warps over (problem, row, head part) items, item = (problem *
+// rows_per_problem_max + row) * hsplit + part (items past a problem's row count are
+// skipped).  A row's head vectors are cut into hsplit parts of hper vectors (whole head
+// passes): one part per row on large batches, several on small ones, so that the rows of a
+// small batch still spread over every warp instead of each warp walking all of its row's
+// passes one memory round trip after another.  A row's D/2 angles are formed per item (two
+// per lane) and shared through shared memory; a lane then owns eight rotation pairs
+// (i, i + D/2) of one head vector (D/16 lanes per head, 16-byte loads and stores,
+// kRopePasses head passes in flight; the first pass's loads are issued before the angles are
+// formed).  The rotation is rope.cuh's (inverse frequencies from the host).
 template <int D>
 __global__ void __launch_bounds__(kRopeWarps * 32, 3) rope_pack_kernel(
     const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k,
-    const int32_t* __restrict__ pos, AttnParams p, float theta, int32_t rows_per_problem_max, int32_t n_prob,
-    int32_t max_pairs, __nv_bfloat16* __restrict__ qhat, __nv_bfloat16* __restrict__ khat) {
+    const int32_t* __restrict__ pos, AttnParams p, const RopeFreqs<D> freqs, int32_t rows_per_problem_max,
+    int32_t n_prob,
+    int32_t max_pairs, int32_t hsplit, int32_t hper, __nv_bfloat16* __restrict__ qhat,
+    __nv_bfloat16* __restrict__ khat) {
   pdl_enter();
   constexpr int LPH = D / 16;       // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
   __shared__ float s_cs[kRopeWarps][D / 2], s_sn[kRopeWarps][D / 2];
-  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
+  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = freqs.f[threadIdx.x];
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (p.plan && blockIdx.x == 0 && warp == 0) attn_plan_warp(p, n_prob, p.new_rows_extent, max_pairs);
   const int sub = lane % LPH, hoff = lane / LPH;
   const int n_vec = p.h_q + p.h_kv;
-  const int64_t total = static_cast<int64_t>(n_prob) * rows_per_problem_max;
+  const int64_t total = static_cast<int64_t>(n_prob) * rows_per_problem_max * hsplit;
   for (int64_t it = static_cast<int64_t>(blockIdx.x) * kRopeWarps + warp; it < total;
        it += static_cast<int64_t>(gridDim.x) * kRopeWarps) {
-    const int prob = static_cast<int>(it / rows_per_problem_max);
-    const int i = static_cast<int>(it - static_cast<int64_t>(prob) * rows_per_problem_max);
+    const int64_t rit = it / hsplit;
+    const int part = static_cast<int>(it - rit * hsplit);
+    const int prob = static_cast<int>(rit / rows_per_problem_max);
+    const int i = static_cast<int>(rit - static_cast<int64_t>(prob) * rows_per_problem_max);
     const Geom gm = problem_geom(p, prob);
     if (i >= gm.n_new) continue;
-    // each pair's angle once per row (a lane takes pairs lane, lane + 32), shared through shared memory
-    const int32_t ps = pos[p.problems ? gm.new_row + i : i];
+    const int64_t row = gm.new_row + i;
+    const int hbeg = part * hper, hend = min(n_vec, hbeg + hper);
+    const int32_t ps = pos[p.problems ? row : i];
+    uint4 x1[kRopePasses], x2[kRopePasses];
+    auto load_pass = [&](int h0) {
+#pragma unroll
+      for (int u = 0; u < kRopePasses; ++u) {
+        const int h = h0 + u * HPP;
+        if (h < hend) {
+          const __nv_bfloat16* src = h < p.h_q ? q + (row * p.h_q + h) * D : k + (row * p.h_kv + (h - p.h_q)) * D;
+          x1[u] = *reinterpret_cast<const uint4*>(src + 8 * sub);
+          x2[u] = *reinterpret_cast<const uint4*>(src + D / 2 + 8 * sub);
+        }
+      }
+    };
+    load_pass(hbeg + hoff);
+    // each pair's angle once per item (a lane takes pairs lane, lane + 32), shared through shared memory
     __syncwarp();
 #pragma unroll
     for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, inv_freq[t], s_sn[warp][t], s_cs[warp][t]);
@@ -189,26 +212,16 @@ __global__ void __launch_bounds__(kRopeWarps * 32, 3) rope_pack_kernel(
       sn0[t] = s_sn[warp][8 * sub + t];
       sn1[t] = s_sn[warp][8 * sub + 4 + t];
     }
-    const int64_t row = gm.new_row + i;
     // a packed unit's softmax rows read their problem's key bounds from here in one load: the
     // cache prefix length and the problem's new rows [new_row, new_row + n_new)
-    if (p.row_bounds && lane == 0)
+    if (p.row_bounds && part == 0 && lane == 0)
       p.row_bounds[row] = make_int4(gm.n_cache, static_cast<int>(gm.new_row), static_cast<int>(gm.new_row + gm.n_new), 0);
-    for (int h0 = hoff; h0 < n_vec; h0 += kRopePasses * HPP) {
-      uint4 x1[kRopePasses], x2[kRopePasses];
+    for (int h0 = hbeg + hoff; h0 < hend; h0 += kRopePasses * HPP) {
+      if (h0 != hbeg + hoff) load_pass(h0);
 #pragma unroll
       for (int u = 0; u < kRopePasses; ++u) {
         const int h = h0 + u * HPP;
-        if (h < n_vec) {
-          const __nv_bfloat16* src = h < p.h_q ? q + (row * p.h_q + h) * D : k + (row * p.h_kv + (h - p.h_q)) * D;
-          x1[u] = *reinterpret_cast<const uint4*>(src + 8 * sub);
-          x2[u] = *reinterpret_cast<const uint4*>(src + D / 2 + 8 * sub);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kRopePasses; ++u) {
-        const int h = h0 + u * HPP;
-        if (h >= n_vec) continue;
+        if (h >= hend) continue;
         uint2 ya, yb, yc, yd;
         rope_rotate4(make_uint2(x1[u].x, x1[u].y), make_uint2(x2[u].x, x2[u].y), cs0, sn0, ya, yb);
         rope_rotate4(make_uint2(x1[u].z, x1[u].w), make_uint2(x2[u].z, x2[u].w), cs1, sn1, yc, yd);
@@ -1029,16 +1042,22 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
   p.wait_ns = wait_limit_ns();
   const int n_prob = batch_or_np;
   if (part != kPartCore) {
-    const int64_t items = static_cast<int64_t>(n_prob) * max_n_new;
     // persistent: as many CTAs per SM as fit (three at the kernel's register bound)
     static const int per_sm = resident_ctas(rope_pack_kernel<D>, kRopeWarps * 32, 0);
-    const int grid = static_cast<int>(
-        std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, static_cast<int64_t>(per_sm) * num_sms()));
+    const int64_t warps = static_cast<int64_t>(per_sm) * num_sms() * kRopeWarps;
+    const int64_t rows = static_cast<int64_t>(n_prob) * max_n_new;
+    // head parts per row: enough items for every warp when the batch has fewer rows than warps,
+    // each part whole passes of kRopePasses x (32 / (D / 16)) head vectors
+    const int pass_vecs = kRopePasses * (32 / (D / 16));
+    const int n_pass = (h_q + h_kv + pass_vecs - 1) / pass_vecs;
+    const int want = static_cast<int>(std::min<int64_t>((warps + rows - 1) / rows, n_pass));
+    const int hper = ((n_pass + want - 1) / want) * pass_vecs;
+    const int hsplit = (h_q + h_kv + hper - 1) / hper;
+    const int64_t items = rows * hsplit;
+    const int grid = static_cast<int>(std::min<int64_t>((items + kRopeWarps - 1) / kRopeWarps, warps / kRopeWarps));
     ssm::launch_k(rope_pack_kernel<D>, dim3(grid), dim3(kRopeWarps * 32), 0, st,
-             static_cast<const __nv_bfloat16*>(q),
-                                                          static_cast<const __nv_bfloat16*>(k_new), pos, p,
-                                                          rope_theta, max_n_new, n_prob, wl.max_pairs, qhat,
-                                                          khat);
+                  static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k_new), pos, p,
+                  rope_freqs<D>(rope_theta), max_n_new, n_prob, wl.max_pairs, hsplit, hper, qhat, khat);
     const ssm_status s = launch_status();
     if (s != SSM_OK || part == kPartRotate) return s;
   }

@@ -25,7 +25,7 @@ constexpr int kAppendWarps = 8;
 template <int D>
 __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
     const __nv_bfloat16* __restrict__ k_new, const __nv_bfloat16* __restrict__ v_new,
-    const int32_t* __restrict__ pos, int32_t batch, int32_t n_rows, int32_t h_kv, float theta,
+    const int32_t* __restrict__ pos, int32_t batch, int32_t n_rows, int32_t h_kv, const RopeFreqs<D> freqs,
     __nv_bfloat16* __restrict__ k_cache, __nv_bfloat16* __restrict__ v_cache, int64_t cache_rows,
     int64_t start_row) {
   pdl_enter();
@@ -33,7 +33,7 @@ __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
   constexpr int HPP = 32 / LPH;  // head vectors per warp pass
   __shared__ double inv_freq[D / 2];
   __shared__ float s_cs[kAppendWarps][D / 2], s_sn[kAppendWarps][D / 2];
-  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = rope_inv_freq(theta, threadIdx.x, D);
+  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = freqs.f[threadIdx.x];
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane % LPH, hoff = lane / LPH;
@@ -116,13 +116,11 @@ ssm_status ssm_cache_append(const void* k_new, const void* v_new, const int32_t*
   auto* kc = static_cast<__nv_bfloat16*>(k_cache);
   auto* vc = static_cast<__nv_bfloat16*>(v_cache);
   if (head_dim == 128)
-    ssm::launch_k(ssm::cache_append_kernel<128>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st,
-             kn, vn, pos, batch, n_rows, h_kv, rope_theta,
-                                                                         kc, vc, cache_rows, start_row);
+    ssm::launch_k(ssm::cache_append_kernel<128>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st, kn, vn, pos,
+                  batch, n_rows, h_kv, ssm::rope_freqs<128>(rope_theta), kc, vc, cache_rows, start_row);
   else
-    ssm::launch_k(ssm::cache_append_kernel<64>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st,
-             kn, vn, pos, batch, n_rows, h_kv, rope_theta,
-                                                                        kc, vc, cache_rows, start_row);
+    ssm::launch_k(ssm::cache_append_kernel<64>, dim3(grid), dim3(ssm::kAppendWarps * 32), 0, st, kn, vn, pos,
+                  batch, n_rows, h_kv, ssm::rope_freqs<64>(rope_theta), kc, vc, cache_rows, start_row);
   return ssm::launch_status();
 }
 

@@ -7,6 +7,7 @@
 
 #include <cuda_bf16.h>
 
+#include <cmath>
 #include <cstdint>
 
 namespace ssm {
@@ -16,9 +17,22 @@ __device__ __forceinline__ uint32_t rope_pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// theta^(-2i/D) in fp64 (0 when theta == 0: no rotation).
-__device__ __forceinline__ double rope_inv_freq(float theta, int i, int d) {
-  return theta > 0.f ? exp2(-(2.0 * i / d) * log2(static_cast<double>(theta))) : 0.0;
+// The D/2 inverse frequencies theta^(-2i/D) in fp64 (all 0 when theta == 0: no
+// rotation).  They are formed on the host, once per launch, and passed to the
+// kernels by value: GB300's fp64 rate is a small fraction of its fp32 rate, and
+// the fp64 exponential and logarithm of every CTA's table were a visible part of
+// a small launch.
+template <int D>
+struct RopeFreqs {
+  double f[D / 2];
+};
+
+template <int D>
+inline RopeFreqs<D> rope_freqs(float theta) {
+  RopeFreqs<D> r;
+  const double l2 = theta > 0.f ? std::log2(static_cast<double>(theta)) : 0.0;
+  for (int i = 0; i < D / 2; ++i) r.f[i] = theta > 0.f ? std::exp2(-(2.0 * i / D) * l2) : 0.0;
+  return r;
 }
 
 // sin and cos of pos * inv_freq: the angle is formed and reduced modulo 2 pi in

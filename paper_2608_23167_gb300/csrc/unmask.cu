@@ -3,21 +3,21 @@
 // ssm_unmask_topk, which also enqueues the retained suffix positions' top-k
 // (topk.cu) for the next step's Eq. 6.
 //
-// Pass 1 (unmask_stream_kernel): every masked row of logits is cut into
-// segments of whole 16 KB chunks (the work items, dealt round-robin to
-// persistent CTAs, three per SM, one wave): one segment per row once a call has
-// 912 rows, shorter ones for smaller calls (about two items per CTA).  Each thread streams its own 64-byte slices of successive
-// 16 KB chunks from HBM into a private two-stage shared-memory ring with
-// 16-byte cp.async copies, so the read runs ahead of the arithmetic without any
-// barrier (a thread only reads back what it copied itself), and folds every
-// chunk into a running (max, first argmax, sum of exp(x - max)) plus, when p2
-// is wanted, the second-largest value.  The 256 running states of a segment are
-// merged into one partial.  Rows whose length or alignment rules out 16-byte
-// copies take unmask_partial_scalar_kernel on the same segment grid.
-// Pass 2 (unmask_commit_kernel): one CTA
-// per batch row merges the segment partials of its positions, writes conf /
-// argmax / p2 and applies the commit rule.  Logits of unmasked rows are never
-// read.
+// Pass 1 (unmask_stream_kernel): the masked rows of logits are cut into 16 KB
+// stages, numbered row-major over the call, and every persistent CTA (three per
+// SM, one wave) takes one contiguous range of the same number of stages, so the
+// CTAs finish together whatever the row length and batch.  Each thread streams
+// its own 64-byte slices of successive stages from HBM into a private two-stage
+// shared-memory ring with 16-byte cp.async copies, so the read runs ahead of the
+// arithmetic without any barrier (a thread only reads back what it copied
+// itself), and folds every stage into a running (max, first argmax, sum of
+// exp(x - max)) plus, when p2 is wanted, the second-largest value.  Where its
+// range leaves a row (or ends), the CTA merges its 256 running states into one
+// partial of that row.  Rows whose length or alignment rules out 16-byte copies
+// take unmask_partial_scalar_kernel on the same ranges.
+// Pass 2 (unmask_commit_kernel): one CTA per batch row merges the partials of
+// its positions (one per CTA whose range meets the row), writes conf / argmax /
+// p2 and applies the commit rule.  Logits of unmasked rows are never read.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -33,7 +33,7 @@ namespace ssm {
 namespace {
 
 constexpr int kUnmaskThreads = 256;
-constexpr int64_t kItemsTarget = 912;              // segments (work items) a call aims for: ~2 per resident CTA
+constexpr int kMaxStreamCtas = 768;                // grid cap of the streaming pass (three CTAs per SM, <= 256 SMs)
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct Partial {
@@ -123,16 +123,6 @@ constexpr int kStageBytes = 16384;                     // one stage: 64 bytes pe
 constexpr int kStreamStages = 2;                       // chunks in flight per thread
 constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
 
-__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("min.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
 
 // Running per-thread state over one segment: max m1 (first index idx), second
 // largest m2 (a repeated maximum counts twice) and s = sum exp(x - m1).
@@ -144,7 +134,7 @@ struct RunState {
 // (three CTAs per SM: the grid is one wave of them)
 template <typename T, bool NEED_SECOND>
 __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
-    const T* __restrict__ logits, int64_t vocab, int64_t seg_elems, int n_seg, int64_t n_rows,
+    const T* __restrict__ logits, int64_t vocab, int32_t n_stage, int64_t per, int64_t n_total, int kr,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
   pdl_enter();
   constexpr int ESZ = sizeof(T);
@@ -154,38 +144,40 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
   uint4* keep = reinterpret_cast<uint4*>(ring + kStreamStages * kStageBytes) + threadIdx.x * kVecPerThread;
   __shared__ Partial wpart[kStreamThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t n_items = n_rows * n_seg;
-  // issue side runs kStreamStages chunks ahead of the compute side; a thread only ever
+  constexpr int64_t SE = kStageBytes / ESZ;  // elements per stage
+  // this CTA's stages [g0, g1)
+  const int64_t g0 = static_cast<int64_t>(blockIdx.x) * per;
+  const int64_t g1 = min(n_total, g0 + per);
+  // issue side runs kStreamStages stages ahead of the compute side; a thread only ever
   // reads the shared-memory bytes it copied itself, so no barrier is needed between them
-  ChunkIter is{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
-  chunk_seek<T>(is, vocab, seg_elems, n_seg, n_items, masked);
+  StageCursor is = stage_begin<T>(g0, g1, n_stage, SE, vocab, masked);
   auto issue = [&](int slot) {
-    if (is.valid) {
-      const uint8_t* src = reinterpret_cast<const uint8_t*>(logits + is.row * vocab + is.e0) + is.off;
+    if (is.g < g1) {
+      const uint8_t* src = reinterpret_cast<const uint8_t*>(logits + is.row * vocab + is.e0);
       uint8_t* dst = ring + slot * kStageBytes;
 #pragma unroll
       for (int u = 0; u < kVecPerThread; ++u) {
         const int vi = u * kStreamThreads + threadIdx.x;
-        if (vi * 16 < is.bytes - is.off) cp_async16(dst + vi * 16, src + vi * 16);
+        if (vi * 16 < is.bytes) cp_async16(dst + vi * 16, src + vi * 16);
       }
-      is.off += kStageBytes;
-      chunk_seek<T>(is, vocab, seg_elems, n_seg, n_items, masked);
+      stage_next<T>(is, g1, n_stage, SE, vocab, masked);
     }
     cp_async_commit();
   };
 #pragma unroll
   for (int k = 0; k < kStreamStages; ++k) issue(k);
 
-  ChunkIter cs{static_cast<int64_t>(blockIdx.x) - gridDim.x, 0, 0, 0, 0, false};
-  chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
+  StageCursor cs = stage_begin<T>(g0, g1, n_stage, SE, vocab, masked);
+  // this CTA's slot among the CTAs whose ranges meet a row: 0 for every row but the first
+  const int64_t first_row = g0 / n_stage;
+  const int first_slot = static_cast<int>(blockIdx.x - (first_row * n_stage) / per);
   int slot = 0;
-  while (cs.valid) {
-    const int64_t item = cs.item;
-    const int64_t e0 = cs.e0;
+  while (cs.g < g1) {
+    const int64_t row = cs.row;
     RunState r{-INFINITY, -INFINITY, 0.f, INT_MAX};
-    while (cs.valid && cs.item == item) {
+    while (cs.g < g1 && cs.row == row) {
       cp_async_wait<kStreamStages - 1>();
-      const int chunk_bytes = static_cast<int>(min(static_cast<int64_t>(kStageBytes), cs.bytes - cs.off));
+      const int chunk_bytes = cs.bytes;
       const uint4* sv = reinterpret_cast<const uint4*>(ring + slot * kStageBytes);
       uint4 v[kVecPerThread];
       bool in[kVecPerThread];
@@ -196,7 +188,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
         in[u] = vi * 16 < chunk_bytes;
         v[u] = in[u] ? sv[vi] : make_uint4(ninf, ninf, ninf, ninf);
       }
-      const int64_t base = e0 + cs.off / ESZ;
+      const int64_t base = cs.e0;
       // this thread's values of the chunk as fp32 (entries past a short last chunk are -inf)
       constexpr int PER = kVecPerThread * 16 / ESZ;  // 32 bf16 or 16 fp32 values
       float f[PER];
@@ -252,13 +244,12 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
         }
         r.s += ((sa[0] + sb[0]) + (sa[1] + sb[1])) + ((sa[2] + sb[2]) + (sa[3] + sb[3]));
       }
-      // the slot has been read and used: refill it with the chunk kStreamStages ahead
+      // the slot has been read and used: refill it with the stage kStreamStages ahead
       issue(slot);
       slot = (slot + 1) % kStreamStages;
-      cs.off += kStageBytes;
-      if (cs.off >= cs.bytes) chunk_seek<T>(cs, vocab, seg_elems, n_seg, n_items, masked);
+      stage_next<T>(cs, g1, n_stage, SE, vocab, masked);
     }
-    // block partial of the segment: per-warp shuffles, then warp 0 merges the eight
+    // the CTA's partial of the row: per-warp shuffles, then thread 0 merges the eight
     // the kept chunk: first position of the maximum and, when wanted, its second largest
     if (r.m1 > -INFINITY) {
       const int tbase = r.idx + static_cast<int>(threadIdx.x) * (16 / ESZ);
@@ -290,53 +281,65 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
     if (threadIdx.x == 0) {
       Partial q = wpart[0];
       for (int w2 = 1; w2 < kStreamThreads / 32; ++w2) q = merge(q, wpart[w2]);
-      part[item] = q;
+      // slot of this CTA among the CTAs whose ranges meet the row
+      part[row * kr + (row == first_row ? first_slot : 0)] = q;
     }
     __syncthreads();
   }
   cp_async_wait<0>();
 }
 
-// Rows whose length or alignment rules out 16-byte vectors: one element per
-// thread per step, online (max, second, first index) then the exp sum.
+// Rows whose length or alignment rules out 16-byte vectors: the same stage ranges,
+// one element per thread per step, online (max, second, first index) then the exp sum,
+// for each row the range meets.
 template <typename T>
 __global__ void __launch_bounds__(kUnmaskThreads) unmask_partial_scalar_kernel(
-    const T* __restrict__ logits, int64_t vocab, int64_t chunk, int n_chunks,
+    const T* __restrict__ logits, int64_t vocab, int32_t n_stage, int64_t per, int64_t n_total, int kr,
     const uint8_t* __restrict__ masked, Partial* __restrict__ part) {
   pdl_enter();
-  const int64_t row = blockIdx.y;
-  if (!masked[row]) return;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * chunk;
-  const int64_t c1 = min(vocab, c0 + chunk);
-  const T* x = logits + row * vocab;
-  float m = -INFINITY, m2 = -INFINITY;
-  int idx = INT_MAX;
-  float s = 0.f;
-  for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
-    observe(Vec<T>::scalar(x, e), static_cast<int>(e), m, idx, m2);
-  if (m > -INFINITY) {
-    const float mb = m * kLog2e;
-    for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
-      s += ex2(fmaf(Vec<T>::scalar(x, e), kLog2e, -mb));
-  }
-  Partial p{m, s, idx, m2};
-#pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) p = merge(p, shfl_partial(p, d));
+  constexpr int64_t SE = kStageBytes / static_cast<int64_t>(sizeof(T));
   __shared__ Partial sp[kUnmaskThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) sp[warp] = p;
-  __syncthreads();
-  if (warp == 0) {
-    p = (lane < kUnmaskThreads / 32) ? sp[lane] : Partial{-INFINITY, 0.f, INT_MAX, -INFINITY};
+  const int64_t g0 = static_cast<int64_t>(blockIdx.x) * per;
+  const int64_t g1 = min(n_total, g0 + per);
+  for (int64_t g = g0; g < g1;) {
+    const int64_t row = g / n_stage;
+    const int64_t gr = min(g1, (row + 1) * n_stage);   // this row's stages in the range end here
+    if (masked[row]) {
+      const int64_t c0 = (g - row * n_stage) * SE;
+      const int64_t c1 = min(vocab, (gr - row * n_stage) * SE);
+      const T* x = logits + row * vocab;
+      float m = -INFINITY, m2 = -INFINITY;
+      int idx = INT_MAX;
+      float s = 0.f;
+      for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
+        observe(Vec<T>::scalar(x, e), static_cast<int>(e), m, idx, m2);
+      if (m > -INFINITY) {
+        const float mb = m * kLog2e;
+        for (int64_t e = c0 + threadIdx.x; e < c1; e += kUnmaskThreads)
+          s += ex2(fmaf(Vec<T>::scalar(x, e), kLog2e, -mb));
+      }
+      Partial p{m, s, idx, m2};
 #pragma unroll
-    for (int d = 4; d >= 1; d >>= 1) p = merge(p, shfl_partial(p, d));
-    if (lane == 0) part[row * n_chunks + blockIdx.x] = p;
+      for (int d = 16; d >= 1; d >>= 1) p = merge(p, shfl_partial(p, d));
+      if (lane == 0) sp[warp] = p;
+      __syncthreads();
+      if (warp == 0) {
+        p = (lane < kUnmaskThreads / 32) ? sp[lane] : Partial{-INFINITY, 0.f, INT_MAX, -INFINITY};
+#pragma unroll
+        for (int d = 4; d >= 1; d >>= 1) p = merge(p, shfl_partial(p, d));
+        if (lane == 0) part[row * kr + (static_cast<int64_t>(blockIdx.x) - (row * n_stage) / per)] = p;
+      }
+      __syncthreads();
+    }
+    g = gr;
   }
 }
 
 // One CTA per batch row; thread j owns block position j.
 __global__ void __launch_bounds__(1024) unmask_commit_kernel(
-    int block_len, int n_chunks, const uint8_t* __restrict__ masked, const Partial* __restrict__ part,
+    int block_len, int32_t n_stage, int64_t per, int kr, const uint8_t* __restrict__ masked,
+    const Partial* __restrict__ part,
     int mode, float threshold, int topk, int min_commit, float* __restrict__ conf,
     int32_t* __restrict__ argmax, float* __restrict__ p2_out, uint8_t* __restrict__ commit) {
   pdl_enter();
@@ -356,9 +359,11 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
     const int64_t row = b * block_len + j;
     mj = masked[row] != 0;
     if (mj) {
-      // the row's partials are loaded eight at a time, independently, then merged (a chain
-      // of dependent loads would cost one memory latency per partial)
-      const Partial* pr = part + row * n_chunks;
+      // the row's partials (one per CTA whose stage range meets the row) are loaded eight at
+      // a time, independently, then merged (a chain of dependent loads would cost one memory
+      // latency per partial)
+      const int n_chunks = static_cast<int>((row * n_stage + n_stage - 1) / per - (row * n_stage) / per + 1);
+      const Partial* pr = part + row * kr;
       Partial p = pr[0];
       for (int c0 = 1; c0 < n_chunks; c0 += 8) {
         Partial q[8];
@@ -410,27 +415,29 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
 namespace {
 
 struct UnmaskPlan {
-  int64_t chunk;
-  int n_chunks;
+  int32_t n_stage;  // 16 KB stages per row
+  int64_t per;      // stages per CTA
+  int64_t total;    // stages of the call (rows x n_stage)
+  int grid;         // CTAs
+  int kr;           // partial slots per row: at most this many CTA ranges meet a row
   bool vector;
 };
 
-// Segments are whole 16 KB stages.  A row is cut into the fewest segments that
-// still give about kItemsTarget work items over all rows: one segment per row
-// once there are that many rows (every segment ends in a CTA-wide merge, so
-// fewer, longer segments stream faster), more for small calls so that their
-// rows still spread over the SMs.
-UnmaskPlan plan_unmask(int64_t rows, int64_t vocab, ssm_dtype dtype, const void* logits) {
+// Every CTA takes `per` consecutive stages of the call, per = ceil(total / CTAs) with at
+// most max_ctas CTAs; a row's n_stage stages then meet at most ceil((n_stage - 1) / per) + 1
+// ranges (and never more than n_stage).  Fewer CTAs give longer ranges and fewer slots per
+// row, so the workspace is sized at the grid cap and fits every grid at or below it.
+UnmaskPlan plan_unmask(int64_t rows, int64_t vocab, ssm_dtype dtype, const void* logits, int max_ctas) {
   const int esz = dtype == SSM_DTYPE_BF16 ? 2 : 4;
   UnmaskPlan p;
   p.vector = ((vocab * esz) % 16 == 0) && (logits == nullptr || ssm::aligned16(logits));
-  // both plans cut a row into the same segments, so the workspace does not depend on the plan
   const int64_t stage_elems = ssm::kStageBytes / esz;
-  const int64_t n_stage = (vocab + stage_elems - 1) / stage_elems;
-  const int64_t per_row = (ssm::kItemsTarget + rows - 1) / std::max<int64_t>(rows, 1);
-  const int64_t want = std::min<int64_t>(std::max<int64_t>(per_row, 1), n_stage);
-  p.chunk = ((n_stage + want - 1) / want) * stage_elems;
-  p.n_chunks = static_cast<int>((vocab + p.chunk - 1) / p.chunk);
+  p.n_stage = static_cast<int32_t>((vocab + stage_elems - 1) / stage_elems);
+  p.total = rows * p.n_stage;
+  const int64_t g = std::max<int64_t>(1, std::min<int64_t>(max_ctas, p.total));
+  p.per = (p.total + g - 1) / g;
+  p.grid = static_cast<int>((p.total + p.per - 1) / p.per);
+  p.kr = static_cast<int>(std::min<int64_t>(p.n_stage, (p.n_stage - 1 + p.per - 1) / p.per + 1));
   return p;
 }
 
@@ -456,8 +463,9 @@ extern "C" {
 
 size_t ssm_unmask_workspace_size(int32_t batch, int32_t block_len, int64_t vocab, ssm_dtype dtype) {
   if (batch <= 0 || block_len <= 0 || vocab <= 0) return 0;
-  const UnmaskPlan plan = plan_unmask(static_cast<int64_t>(batch) * block_len, vocab, dtype, nullptr);
-  return ssm::align_up(static_cast<size_t>(batch) * block_len * plan.n_chunks * sizeof(ssm::Partial), 256);
+  const UnmaskPlan plan =
+      plan_unmask(static_cast<int64_t>(batch) * block_len, vocab, dtype, nullptr, ssm::kMaxStreamCtas);
+  return ssm::align_up(static_cast<size_t>(batch) * block_len * plan.kr * sizeof(ssm::Partial), 256);
 }
 
 ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_t block_len,
@@ -478,15 +486,14 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   if (ws_bytes < ssm_unmask_workspace_size(batch, block_len, vocab, dtype)) return SSM_ERR_CAPACITY;
   const int64_t rows = static_cast<int64_t>(batch) * block_len;
   if (rows > 65535) return SSM_ERR_UNSUPPORTED;
-  const UnmaskPlan plan = plan_unmask(rows, vocab, dtype, logits);
+  // one wave: three CTAs per SM are resident (registers)
+  const UnmaskPlan plan =
+      plan_unmask(rows, vocab, dtype, logits, std::min(3 * ssm::num_sms(), ssm::kMaxStreamCtas));
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  dim3 grid(plan.n_chunks, static_cast<unsigned>(rows));
   // the ring (32 KB) and a 64-byte copy per thread of its maximum's chunk (16 KB)
   const size_t stream_smem = (ssm::kStreamStages + 1) * ssm::kStageBytes + 128;
-  const int64_t n_items = rows * plan.n_chunks;
-  // one wave: three CTAs per SM are resident (registers), each takes ~2 items of ~kItemsTarget
-  const int stream_grid = static_cast<int>(std::min<int64_t>(n_items, 3 * ssm::num_sms()));
+  const int stream_grid = plan.grid;
   const bool need_second = p2 != nullptr || mode == SSM_COMMIT_MARGIN;
   if (dtype == SSM_DTYPE_BF16) {
     auto* x = static_cast<const __nv_bfloat16*>(logits);
@@ -496,13 +503,13 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
         return SSM_ERR_CUDA;
       if (need_second)
         ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
     } else {
-      ssm::launch_k(ssm::unmask_partial_scalar_kernel<__nv_bfloat16>, dim3(grid), dim3(ssm::kUnmaskThreads), 0, st,
-               x, vocab, plan.chunk, plan.n_chunks, masked, part);
+      ssm::launch_k(ssm::unmask_partial_scalar_kernel<__nv_bfloat16>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0,
+                    st, x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
     }
   } else {
     auto* x = static_cast<const float*>(logits);
@@ -512,13 +519,13 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
         return SSM_ERR_CUDA;
       if (need_second)
         ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
       else
         ssm::launch_k(ssm::unmask_stream_kernel<float, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.chunk, plan.n_chunks, rows, masked, part);
+                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
     } else {
-      ssm::launch_k(ssm::unmask_partial_scalar_kernel<float>, dim3(grid), dim3(ssm::kUnmaskThreads), 0, st,
-               x, vocab, plan.chunk, plan.n_chunks, masked, part);
+      ssm::launch_k(ssm::unmask_partial_scalar_kernel<float>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0, st,
+                    x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
     }
   }
   ssm_status s = ssm::launch_status();
@@ -526,7 +533,7 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   const int threads = ((block_len + 31) / 32) * 32;
   const size_t shm = static_cast<size_t>(block_len) * (2 * sizeof(float) + 2);
   ssm::launch_k(ssm::unmask_commit_kernel, dim3(batch), dim3(threads), shm, st,
-           block_len, plan.n_chunks, masked, part, mode,
+           block_len, plan.n_stage, plan.per, plan.kr, masked, part, mode,
                                                          threshold, topk, min_commit, conf, argmax, p2,
                                                          commit);
   return ssm::launch_status();
@@ -583,10 +590,11 @@ ssm_status ssm_unmask_topk(const void* logits, ssm_dtype dtype, int32_t batch, i
 
 namespace {
 
-// 1 MiB holds 65536 chunk partials: e.g. 512 sequences x 32 positions x 4
-// chunks of a 126464-entry bf16 vocabulary.  Every GPU that loads libssm
-// keeps this array until the process exits.
-constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;
+// 2 MiB holds 131072 16-byte row partials: two per row for every call of up to
+// 65535 positions of a 126464-entry bf16 or fp32 vocabulary (more per row only
+// for calls with fewer rows than the streaming pass has CTAs).  Every GPU that
+// loads libssm keeps this array until the process exits.
+constexpr size_t kNoAllocScratchBytes = size_t(2) << 20;
 static __device__ __align__(256) unsigned char g_unmask_scratch[kNoAllocScratchBytes];
 
 constexpr int kMaxDevices = 64;
@@ -622,7 +630,7 @@ extern "C" ssm_status ssm_unmask_noalloc(const void* logits, ssm_dtype dtype, in
   void* scratch = nullptr;
   const ssm_status s = scratch_address(&scratch);
   if (s != SSM_OK) return s;
-  // The chunk partials are written before they are read on every call, so the
+  // The row partials are written before they are read on every call, so the
   // previous call's contents never need clearing.
   return ssm_unmask(logits, dtype, batch, block_len, vocab, masked, mode, threshold, topk, min_commit, conf,
                     argmax, p2, commit, scratch, kNoAllocScratchBytes, stream);

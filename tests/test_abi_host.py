@@ -118,11 +118,15 @@ def test_workspace_sizes(lib):
     rows, pairs = 8854, (8854 * 7 + 255) // 256    # GQA: 7 query heads per kv head pack 7 rows per query
     assert ssm.ssm_attention_workspace_size(rows, 28, 4, 128) == (
         up(rows * 28 * 256) + up(rows * 4 * 256) + up(32 + 32 * pairs) + up(16 * rows))
-    # 126464 bf16 entries are 16 stages of 8192; segments aim at 912 work items per call
+    # 126464 bf16 entries are 16 stages of 8192; sized at the grid cap of 768 CTAs, each taking
+    # per = ceil(stages / 768) consecutive stages, a row meets at most ceil(15 / per) + 1 CTA
+    # ranges (at most 16), one 16-byte partial each
     ws = ssm.ssm_unmask_workspace_size(8, 32, 126464, torch.bfloat16)
-    assert ws == 8 * 32 * 4 * 16   # 256 rows: four segments of four stages each, 16-byte partials
-    assert ssm.ssm_unmask_workspace_size(64, 32, 126464, torch.bfloat16) == 64 * 32 * 16   # one segment per row
-    assert ssm.ssm_unmask_workspace_size(1, 4, 126464, torch.bfloat16) == 4 * 16 * 16      # one stage per segment
+    assert ws == 8 * 32 * 4 * 16   # 4096 stages: per = 6, four ranges per row
+    assert ssm.ssm_unmask_workspace_size(64, 32, 126464, torch.bfloat16) == 64 * 32 * 2 * 16   # per = 43: two
+    assert ssm.ssm_unmask_workspace_size(1, 4, 126464, torch.bfloat16) == 4 * 16 * 16      # per = 1: sixteen
+    # fp32 rows of 4096 entries are one stage: one partial per row
+    assert ssm.ssm_unmask_workspace_size(1, 32, 4096, torch.float32) == 32 * 16
 
 
 def test_attention_digest_covers_its_includes():

@@ -56,8 +56,9 @@ def test_unmask_noalloc_rejects_sizes_beyond_its_scratch():
     build_lib.build()
     lib = ssm.lib()
     fake = 1 << 20
-    # from 2048 positions on, each 126464-entry bf16 row is one segment with one 16-byte partial:
-    # 65536 positions fill 1 MiB exactly, one more does not fit
-    assert lib.ssm_unmask_workspace_size(2048, 32, 126464, 0) == 1 << 20
+    # with this many positions every streaming range covers more than a row of a 126464-entry
+    # bf16 vocabulary, so a row meets at most two ranges (two 16-byte partials): 65536
+    # positions fill 2 MiB exactly, one sequence more does not fit (and nothing is enqueued)
+    assert lib.ssm_unmask_workspace_size(2048, 32, 126464, 0) == 2 << 20
     assert lib.ssm_unmask_noalloc(fake, 0, 2049, 32, 126464, fake, 0, ctypes.c_float(0.9), 1, 1, fake, fake,
                                   fake, fake, None) == 3
