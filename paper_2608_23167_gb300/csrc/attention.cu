@@ -166,9 +166,9 @@ __global__ void __launch_bounds__(kRopeWarps * 32, 3) rope_pack_kernel(
   pdl_enter();
   constexpr int LPH = D / 16;       // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;     // head vectors per warp pass
-  __shared__ double inv_freq[D / 2];
+  __shared__ uint64_t turn[D / 2];
   __shared__ float s_cs[kRopeWarps][D / 2], s_sn[kRopeWarps][D / 2];
-  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = freqs.f[threadIdx.x];
+  if (threadIdx.x < D / 2) turn[threadIdx.x] = freqs.turn[threadIdx.x];
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (p.plan && blockIdx.x == 0 && warp == 0) attn_plan_warp(p, n_prob, p.new_rows_extent, max_pairs);
@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(kRopeWarps * 32, 3) rope_pack_kernel(
     // each pair's angle once per item (a lane takes pairs lane, lane + 32), shared through shared memory
     __syncwarp();
 #pragma unroll
-    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, inv_freq[t], s_sn[warp][t], s_cs[warp][t]);
+    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, turn[t], s_sn[warp][t], s_cs[warp][t]);
     __syncwarp();
     float cs0[4], cs1[4], sn0[4], sn1[4];
 #pragma unroll

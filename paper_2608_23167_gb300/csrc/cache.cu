@@ -31,9 +31,9 @@ __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
   pdl_enter();
   constexpr int LPH = D / 16;    // lanes per head vector: eight rotation pairs per lane
   constexpr int HPP = 32 / LPH;  // head vectors per warp pass
-  __shared__ double inv_freq[D / 2];
+  __shared__ uint64_t turn[D / 2];
   __shared__ float s_cs[kAppendWarps][D / 2], s_sn[kAppendWarps][D / 2];
-  if (threadIdx.x < D / 2) inv_freq[threadIdx.x] = freqs.f[threadIdx.x];
+  if (threadIdx.x < D / 2) turn[threadIdx.x] = freqs.turn[threadIdx.x];
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane % LPH, hoff = lane / LPH;
@@ -47,7 +47,7 @@ __global__ void __launch_bounds__(kAppendWarps * 32) cache_append_kernel(
     const int32_t ps = pos[i];
     __syncwarp();
 #pragma unroll
-    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, inv_freq[t], s_sn[warp][t], s_cs[warp][t]);
+    for (int t = lane; t < D / 2; t += 32) rope_sincos(ps, turn[t], s_sn[warp][t], s_cs[warp][t]);
     __syncwarp();
     float cs0[4], cs1[4], sn0[4], sn1[4];
 #pragma unroll
