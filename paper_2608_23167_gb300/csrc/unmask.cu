@@ -120,7 +120,7 @@ struct Vec<float> {
 
 constexpr int kStreamThreads = 256;
 constexpr int kStageBytes = 16384;                     // one stage: 64 bytes per thread
-constexpr int kStreamStages = 2;                       // chunks in flight per thread
+constexpr int kStreamStages = 2;                       // stages in flight per thread
 constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
 
 
@@ -357,22 +357,23 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
   bool mj = false;
   if (j < block_len) {
     const int64_t row = b * block_len + j;
+    // the row's partials (one per CTA whose stage range meets the row) are loaded eight at a
+    // time, independently, then merged (a chain of dependent loads would cost one memory
+    // latency per partial), and they are loaded together with the row's mask byte: an
+    // unmasked row's slots hold no partial of this call, and what they hold is not used
+    const int n_chunks = static_cast<int>((row * n_stage + n_stage - 1) / per - (row * n_stage) / per + 1);
+    const Partial* pr = part + row * kr;
+    Partial p = pr[0];
     mj = masked[row] != 0;
+    for (int c0 = 1; c0 < n_chunks; c0 += 8) {
+      Partial q[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) q[c] = pr[min(c0 + c, n_chunks - 1)];
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (c0 + c < n_chunks) p = merge(p, q[c]);
+    }
     if (mj) {
-      // the row's partials (one per CTA whose stage range meets the row) are loaded eight at
-      // a time, independently, then merged (a chain of dependent loads would cost one memory
-      // latency per partial)
-      const int n_chunks = static_cast<int>((row * n_stage + n_stage - 1) / per - (row * n_stage) / per + 1);
-      const Partial* pr = part + row * kr;
-      Partial p = pr[0];
-      for (int c0 = 1; c0 < n_chunks; c0 += 8) {
-        Partial q[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) q[c] = pr[min(c0 + c, n_chunks - 1)];
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          if (c0 + c < n_chunks) p = merge(p, q[c]);
-      }
       const float inv = 1.f / p.s;                     // largest probability = 1 / sum exp(x - max)
       cj = inv;
       p2 = (p.m2 > -INFINITY) ? ex2((p.m2 - p.m) * kLog2e) * inv : 0.f;
@@ -457,6 +458,26 @@ bool stream_attr_set(size_t bytes) {
   return true;
 }
 
+// One streaming launch: the kernel form for the dtype and p2 tracking.  The ring (two 16 KB
+// stages) and a 64-byte copy per thread of its maximum's stage (16 KB) exceed the default
+// 48 KB of dynamic shared memory.
+template <typename T, bool NEED_SECOND>
+ssm_status launch_stream_form(int grid, cudaStream_t st, const T* x, int64_t vocab, const UnmaskPlan& plan,
+                              const uint8_t* masked, ssm::Partial* part) {
+  const size_t smem = (ssm::kStreamStages + 1) * ssm::kStageBytes + 128;
+  if (!stream_attr_set<ssm::unmask_stream_kernel<T, NEED_SECOND>>(smem)) return SSM_ERR_CUDA;
+  ssm::launch_k(ssm::unmask_stream_kernel<T, NEED_SECOND>, dim3(grid), dim3(ssm::kStreamThreads), smem, st, x, vocab,
+                plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
+  return SSM_OK;
+}
+
+template <typename T>
+ssm_status launch_stream(const T* x, bool need_second, int grid, cudaStream_t st, int64_t vocab,
+                         const UnmaskPlan& plan, const uint8_t* masked, ssm::Partial* part) {
+  return need_second ? launch_stream_form<T, true>(grid, st, x, vocab, plan, masked, part)
+                     : launch_stream_form<T, false>(grid, st, x, vocab, plan, masked, part);
+}
+
 }  // namespace
 
 extern "C" {
@@ -491,42 +512,21 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
       plan_unmask(rows, vocab, dtype, logits, std::min(3 * ssm::num_sms(), ssm::kMaxStreamCtas));
   auto* part = static_cast<ssm::Partial*>(workspace);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // the ring (32 KB) and a 64-byte copy per thread of its maximum's chunk (16 KB)
-  const size_t stream_smem = (ssm::kStreamStages + 1) * ssm::kStageBytes + 128;
   const int stream_grid = plan.grid;
   const bool need_second = p2 != nullptr || mode == SSM_COMMIT_MARGIN;
-  if (dtype == SSM_DTYPE_BF16) {
-    auto* x = static_cast<const __nv_bfloat16*>(logits);
-    if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, true>>(stream_smem) ||
-          !stream_attr_set<ssm::unmask_stream_kernel<__nv_bfloat16, false>>(stream_smem))
-        return SSM_ERR_CUDA;
-      if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-      else
-        ssm::launch_k(ssm::unmask_stream_kernel<__nv_bfloat16, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-    } else {
-      ssm::launch_k(ssm::unmask_partial_scalar_kernel<__nv_bfloat16>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0,
-                    st, x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-    }
+  if (plan.vector) {
+    const ssm_status s0 = dtype == SSM_DTYPE_BF16
+        ? launch_stream(static_cast<const __nv_bfloat16*>(logits), need_second, stream_grid, st, vocab, plan, masked,
+                        part)
+        : launch_stream(static_cast<const float*>(logits), need_second, stream_grid, st, vocab, plan, masked, part);
+    if (s0 != SSM_OK) return s0;
+  } else if (dtype == SSM_DTYPE_BF16) {
+    ssm::launch_k(ssm::unmask_partial_scalar_kernel<__nv_bfloat16>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0,
+                  st, static_cast<const __nv_bfloat16*>(logits), vocab, plan.n_stage, plan.per, plan.total, plan.kr,
+                  masked, part);
   } else {
-    auto* x = static_cast<const float*>(logits);
-    if (plan.vector) {
-      if (!stream_attr_set<ssm::unmask_stream_kernel<float, true>>(stream_smem) ||
-          !stream_attr_set<ssm::unmask_stream_kernel<float, false>>(stream_smem))
-        return SSM_ERR_CUDA;
-      if (need_second)
-        ssm::launch_k(ssm::unmask_stream_kernel<float, true>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-      else
-        ssm::launch_k(ssm::unmask_stream_kernel<float, false>, dim3(stream_grid), dim3(ssm::kStreamThreads), stream_smem, st,
-                 x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-    } else {
-      ssm::launch_k(ssm::unmask_partial_scalar_kernel<float>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0, st,
-                    x, vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
-    }
+    ssm::launch_k(ssm::unmask_partial_scalar_kernel<float>, dim3(stream_grid), dim3(ssm::kUnmaskThreads), 0, st,
+                  static_cast<const float*>(logits), vocab, plan.n_stage, plan.per, plan.total, plan.kr, masked, part);
   }
   ssm_status s = ssm::launch_status();
   if (s != SSM_OK) return s;

@@ -183,3 +183,33 @@ def test_unmask_commit_positions_separated(dev, mode, threshold, topk, min_commi
     exact = _check_commits(conf_r, p2_r, masked.numpy(), commit, commit_r, md, threshold, topk, min_commit)
     assert exact == batch
     assert np.array_equal(commit, commit_r)
+
+
+@pytest.mark.parametrize("mode,threshold,want_p2", [("threshold", 0.9, False), ("margin", 0.5, True)])
+def test_unmask_long_sweep_full_size_sampled(dev, mode, threshold, want_p2):
+    """The long-sequence sweep's unmasking at full size, in the launch configuration the bench
+    times: 64 sequences x 32 masked positions x 126464 bf16 logits ~ N(0, 4^2) (518 MB, CTA
+    stage ranges that span several rows; the threshold rule without p2, as the bench calls it).
+    The oracle checks four sampled sequences (their commits depend only on their own 32
+    positions)."""
+    from paper_2608_23167_gb300 import ssm
+    batch, B, V = 64, 32, W.LLADA_VOCAB
+    logits = W.draw_logits((batch, B, V), "bf16", 4.0, seed=64, planted_frac=0.1)
+    masked = torch.ones((batch, B), dtype=torch.uint8)
+    md = MODES[mode]
+    conf = torch.full((batch, B), -1.0, device=dev)
+    arg = torch.full((batch, B), -5, dtype=torch.int32, device=dev)
+    commit = torch.full((batch, B), 9, dtype=torch.uint8, device=dev)
+    p2 = torch.full((batch, B), -1.0, device=dev) if want_p2 else None
+    ssm.ssm_unmask(logits.to(dev), masked.to(dev), conf, arg, commit, p2=p2, mode=md, threshold=threshold,
+                   topk=1, min_commit=1)
+    torch.cuda.synchronize()
+    check_device_error()
+    conf, arg, commit = conf.cpu().double().numpy(), arg.cpu().numpy(), commit.cpu().numpy()
+    for s in (0, 21, 42, 63):
+        conf_r, arg_r, p2_r, commit_r = O.unmask(f64(logits[s:s + 1]), masked[s:s + 1].numpy(), md, threshold, 1, 1)
+        assert np.array_equal(arg[s:s + 1], arg_r), f"sequence {s}"
+        assert np.allclose(conf[s:s + 1], conf_r, rtol=1e-5, atol=0), f"sequence {s}"
+        if want_p2:
+            assert np.allclose(p2[s:s + 1].cpu().double().numpy(), p2_r, rtol=1e-5, atol=1e-30), f"sequence {s}"
+        _check_commits(conf_r, p2_r, masked[s:s + 1].numpy(), commit[s:s + 1], commit_r, md, threshold, 1, 1)
