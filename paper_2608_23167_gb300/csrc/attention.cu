@@ -324,12 +324,12 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
     w.gm = problem_geom(p, w.prob);
     const int rows_q = w.gm.n_new * p.grp;
     const int n_qt = (rows_q + kBM - 1) / kBM;
-    w.qt0 = 2 * pair;
+    w.qt0 = p.tiles_per_unit * pair;
     w.urows = rows_q - w.qt0 * kBM;
     w.orow0 = w.gm.new_row * p.grp + w.qt0 * kBM;
     w.qrow0 = w.orow0;
     w.valid = w.qt0 < n_qt;
-    w.two = w.qt0 + 1 < n_qt;
+    w.two = p.tiles_per_unit == 2 && w.qt0 + 1 < n_qt;
     w.packed = false;
   }
   w.n_csub = (w.gm.n_cache + kSub - 1) / kSub;
@@ -1062,7 +1062,20 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     if (s != SSM_OK || part == kPartRotate) return s;
   }
   const int m_tiles = static_cast<int>((static_cast<int64_t>(max_n_new) * grp + kBM - 1) / kBM);
-  p.units_per_pg = (m_tiles + 1) / 2;
+  // Problem units hold a pair of query tiles (both slots on every key tile) or, when that leaves
+  // most SMs idle, single tiles (the slots split the key tiles and merge): the choice with the
+  // shorter estimated makespan, in key tiles per slot chain, rounds of units x chain per unit
+  // (a single tile's chain is half its key tiles plus about one tile for the merge).
+  {
+    const int64_t nt = ((static_cast<int64_t>(max_n_cache) + kSub - 1) / kSub +
+                        (static_cast<int64_t>(max_n_new) + kSub - 1) / kSub + 3) / 4;
+    const int64_t pgs = static_cast<int64_t>(n_prob) * h_kv;
+    const int64_t sms = num_sms();
+    const int64_t pair_cost = ((pgs * ((m_tiles + 1) / 2) + sms - 1) / sms) * nt;
+    const int64_t single_cost = ((pgs * m_tiles + sms - 1) / sms) * ((nt + 1) / 2 + 1);
+    p.tiles_per_unit = single_cost < pair_cost ? 1 : 2;
+  }
+  p.units_per_pg = p.tiles_per_unit == 2 ? (m_tiles + 1) / 2 : m_tiles;
   const int64_t total_units = static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
   if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
   p.total_units = static_cast<int32_t>(total_units);

@@ -60,6 +60,7 @@ struct AttnParams {
   AttnPlanHdr* plan;                 // ragged batches: the unit plan (header, then units), else null
   int4* row_bounds;                  // ragged batches: per new row, its problem's (n_cache, new_row, new_row + n_new)
   int32_t units_per_pg;              // work units per (problem, kv head)
+  int32_t tiles_per_unit;            // problem units: 128-row query tiles per unit (2: a pair, 1: single tiles)
   int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)
   __nv_bfloat16* out;
