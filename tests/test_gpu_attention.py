@@ -80,31 +80,82 @@ def test_attention_matches_oracle(dev, batch, n_new, n_cache, h_q, h_kv, d, thet
 
 
 def test_attention_full_workloads_sampled(dev):
-    """Full-size serving and Dream launches; the oracle checks a sample of heads."""
+    """Full-size serving, Dream and LLaDA launches (the serving batch's one-tile problems, Dream's
+    single-tile units, LLaDA's pairs of query tiles over 32 heads without a cache); the oracle
+    checks a sample of heads."""
     from paper_2608_23167_gb300 import ssm
-    for name in ("serve", "dream"):
+    for name in ("serve", "dream", "llada"):
         w = W.WORKLOADS[name]
         r, *_ = O.select_suffix(w.prompt, w.gen, w.block, 0, w.local, w.middle, w.tail)
-        n_new = w.block + len(r)
-        pos = torch.tensor(list(range(W.block_start(w, 0), W.block_start(w, 0) + w.block)) + r, dtype=torch.int32)
-        out, ref_unused, lse, _ = None, None, None, None
+        n_cache = w.prompt if w.prefix_cached else 0
+        # without a cache the step recomputes the prompt: its rows come first, at positions 0..P-1
+        prefix = [] if w.prefix_cached else list(range(w.prompt))
+        bs = W.block_start(w, 0)
+        plist = prefix + list(range(bs, bs + w.block)) + r
+        n_new = len(plist)
+        pos = torch.tensor(plist, dtype=torch.int32)
         q = W.draw_normal_bf16((w.batch, n_new, w.h_q, w.head_dim), 1.0, 31)
         k = W.draw_normal_bf16((w.batch, n_new, w.h_kv, w.head_dim), 1.0, 32)
         v = W.draw_normal_bf16((w.batch, n_new, w.h_kv, w.head_dim), 1.0, 33)
-        kc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 34)
-        vc = W.draw_normal_bf16((w.batch, w.prompt, w.h_kv, w.head_dim), 1.0, 35)
+        kc = vc = None
+        if n_cache:
+            kc = W.draw_normal_bf16((w.batch, n_cache, w.h_kv, w.head_dim), 1.0, 34)
+            vc = W.draw_normal_bf16((w.batch, n_cache, w.h_kv, w.head_dim), 1.0, 35)
         o = torch.empty((w.batch, n_new, w.h_q, w.head_dim), dtype=torch.bfloat16, device=dev)
-        ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), o, w.rope_theta)
+        ssm.ssm_attention(q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev) if n_cache else None,
+                          vc.to(dev) if n_cache else None, o, w.rope_theta)
         torch.cuda.synchronize()
         check_device_error()
         grp = w.h_q // w.h_kv
-        for b in (0, w.batch - 1):
-            g = w.h_kv - 1
-            hs = list(range(g * grp, (g + 1) * grp))
-            ref, _ = O.attention(f64(q[b:b + 1, :, hs]), f64(k[b:b + 1, :, g:g + 1]), f64(v[b:b + 1, :, g:g + 1]),
-                                 pos.numpy(), f64(kc[b:b + 1, :, g:g + 1]), f64(vc[b:b + 1, :, g:g + 1]),
+        for b in sorted({0, w.batch - 1}):
+            for g in sorted({0, w.h_kv - 1}):
+                hs = list(range(g * grp, (g + 1) * grp))
+                ref, _ = O.attention(f64(q[b:b + 1, :, hs]), f64(k[b:b + 1, :, g:g + 1]), f64(v[b:b + 1, :, g:g + 1]),
+                                     pos.numpy(), f64(kc[b:b + 1, :, g:g + 1]) if n_cache else None,
+                                     f64(vc[b:b + 1, :, g:g + 1]) if n_cache else None, w.rope_theta)
+                assert_attention_close(f64(o[b:b + 1, :, hs]), ref, f"{name} batch {b} kv head {g}")
+
+
+def test_attention_long_sweep_full_size_sampled(dev):
+    """The long-sequence sweep at full size, in the launch configuration the bench times: the
+    64 block indices over one shared 32-head prefix cache as one ragged launch (packed units
+    over 32 kv heads, rotate and core as two calls); the oracle checks three block indices on
+    three heads."""
+    from paper_2608_23167_gb300 import ssm
+    w = W.WORKLOADS["long"]
+    H, d = w.h_q, w.head_dim
+    total_pos = w.prompt + w.gen
+    kc = W.draw_normal_bf16((total_pos, H, d), 1.0, 51)
+    vc = W.draw_normal_bf16((total_pos, H, d), 1.0, 52)
+    rows, poss, new_row = [], [], 0
+    for b in range(w.n_blocks):
+        r, *_ = O.select_suffix(w.prompt, w.gen, w.block, b, w.local, w.middle, w.tail)
+        bs = W.block_start(w, b)
+        p = list(range(bs, bs + w.block)) + r
+        rows.append((new_row, 0, len(p), bs))
+        poss.extend(p)
+        new_row += len(p)
+    q = W.draw_normal_bf16((new_row, H, d), 1.0, 53)
+    k = W.draw_normal_bf16((new_row, H, d), 1.0, 54)
+    v = W.draw_normal_bf16((new_row, H, d), 1.0, 55)
+    pos = torch.tensor(poss, dtype=torch.int32)
+    probs = ssm.attn_problems_tensor(rows, dev)
+    out = torch.full((new_row, H, d), float("nan"), dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(ssm.ssm_attention_workspace_size(new_row, H, H, d), dtype=torch.uint8, device=dev)
+    args = (q.to(dev), k.to(dev), v.to(dev), pos.to(dev), kc.to(dev), vc.to(dev), probs, len(rows),
+            max(r[2] for r in rows), max(r[3] for r in rows), out, w.rope_theta)
+    ssm.ssm_attention_varlen_rotate(*args, workspace=ws)
+    ssm.ssm_attention_varlen_core(*args, workspace=ws)
+    torch.cuda.synchronize()
+    check_device_error()
+    for b in (0, 31, 63):
+        nr, _, n, nc = rows[b]
+        sl = slice(nr, nr + n)
+        for h in (0, 17, 31):
+            ref, _ = O.attention(f64(q[None, sl, h:h + 1]), f64(k[None, sl, h:h + 1]), f64(v[None, sl, h:h + 1]),
+                                 pos[sl].numpy(), f64(kc[None, :nc, h:h + 1]), f64(vc[None, :nc, h:h + 1]),
                                  w.rope_theta)
-            assert_attention_close(f64(o[b:b + 1, :, hs]), ref, f"{name} batch {b}")
+            assert_attention_close(f64(out[sl, h:h + 1])[None], ref, f"block {b} head {h}")
 
 
 def test_attention_varlen_block_sweep(dev):
