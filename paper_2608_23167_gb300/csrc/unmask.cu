@@ -124,7 +124,7 @@ constexpr int kStreamStages = 2;                       // stages in flight per t
 constexpr int kVecPerThread = kStageBytes / 16 / kStreamThreads;  // 4
 
 
-// Running per-thread state over one segment: max m1 (first index idx), second
+// Running per-thread state over one row's stages in a CTA range: max m1 (first index idx), second
 // largest m2 (a repeated maximum counts twice) and s = sum exp(x - m1).
 struct RunState {
   float m1, m2, s;
@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
   constexpr int ESZ = sizeof(T);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
-  // each thread's copy of its 64 bytes of the chunk that holds its running maximum
+  // each thread's copy of its 64 bytes of the stage that holds its running maximum
   uint4* keep = reinterpret_cast<uint4*>(ring + kStreamStages * kStageBytes) + threadIdx.x * kVecPerThread;
   __shared__ Partial wpart[kStreamThreads / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -177,7 +177,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
     RunState r{-INFINITY, -INFINITY, 0.f, INT_MAX};
     while (cs.g < g1 && cs.row == row) {
       cp_async_wait<kStreamStages - 1>();
-      const int chunk_bytes = cs.bytes;
+      const int stage_bytes = cs.bytes;
       const uint4* sv = reinterpret_cast<const uint4*>(ring + slot * kStageBytes);
       uint4 v[kVecPerThread];
       bool in[kVecPerThread];
@@ -185,11 +185,11 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
 #pragma unroll
       for (int u = 0; u < kVecPerThread; ++u) {
         const int vi = u * kStreamThreads + threadIdx.x;
-        in[u] = vi * 16 < chunk_bytes;
+        in[u] = vi * 16 < stage_bytes;
         v[u] = in[u] ? sv[vi] : make_uint4(ninf, ninf, ninf, ninf);
       }
       const int64_t base = cs.e0;
-      // this thread's values of the chunk as fp32 (entries past a short last chunk are -inf)
+      // this thread's values of the stage as fp32 (entries past a short last stage are -inf)
       constexpr int PER = kVecPerThread * 16 / ESZ;  // 32 bf16 or 16 fp32 values
       float f[PER];
 #pragma unroll
@@ -205,7 +205,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
           }
         }
       }
-      // chunk maximum (four chains of 3-input max) and, when asked for, the second largest
+      // stage maximum (four chains of 3-input max) and, when asked for, the second largest
       float c4[4] = {f[0], f[1], f[2], f[3]};
 #pragma unroll
       for (int e = 4; e < PER; e += 8) {
@@ -218,16 +218,16 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
       }
       const float cm1 = fmaxf(fmaxf(c4[0], c4[1]), fmaxf(c4[2], c4[3]));
       // The argmax (first position of the maximum) and, when wanted, the second largest (a
-      // repeated maximum counts twice) are taken once, at the segment's end, from a copy of the
-      // maximum's chunk: a chunk that raises a lane's maximum only stores its 64 bytes (four
-      // 16-byte shared-memory stores; on most chunks some lane of the warp does).  The second
-      // largest is then the larger of the second largest inside that chunk and the largest
-      // value of every other chunk, which r.m2 keeps.
+      // repeated maximum counts twice) are taken once, where the range leaves the row, from a
+      // copy of the maximum's stage: a stage that raises a lane's maximum only stores its 64
+      // bytes (four 16-byte shared-memory stores; on most stages some lane of the warp does).
+      // The second largest is then the larger of the second largest inside that stage and the
+      // largest value of every other stage, which r.m2 keeps.
       if (cm1 > r.m1) {
         if constexpr (NEED_SECOND) r.m2 = fmaxf(r.m2, r.m1);
 #pragma unroll
         for (int u = 0; u < kVecPerThread; ++u) keep[u] = v[u];
-        r.idx = static_cast<int>(base);   // the kept chunk's first entry
+        r.idx = static_cast<int>(base);   // the kept stage's first entry
         if (r.m1 > -INFINITY) r.s *= ex2((r.m1 - cm1) * kLog2e);
         r.m1 = cm1;
       } else if constexpr (NEED_SECOND) {
@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(kStreamThreads, 3) unmask_stream_kernel(
       stage_next<T>(cs, g1, n_stage, SE, vocab, masked);
     }
     // the CTA's partial of the row: per-warp shuffles, then thread 0 merges the eight
-    // the kept chunk: first position of the maximum and, when wanted, its second largest
+    // the kept stage: first position of the maximum and, when wanted, its second largest
     if (r.m1 > -INFINITY) {
       const int tbase = r.idx + static_cast<int>(threadIdx.x) * (16 / ESZ);
       constexpr int EPV = 16 / ESZ;
@@ -361,17 +361,17 @@ __global__ void __launch_bounds__(1024) unmask_commit_kernel(
     // time, independently, then merged (a chain of dependent loads would cost one memory
     // latency per partial), and they are loaded together with the row's mask byte: an
     // unmasked row's slots hold no partial of this call, and what they hold is not used
-    const int n_chunks = static_cast<int>((row * n_stage + n_stage - 1) / per - (row * n_stage) / per + 1);
+    const int n_part = static_cast<int>((row * n_stage + n_stage - 1) / per - (row * n_stage) / per + 1);
     const Partial* pr = part + row * kr;
     Partial p = pr[0];
     mj = masked[row] != 0;
-    for (int c0 = 1; c0 < n_chunks; c0 += 8) {
+    for (int c0 = 1; c0 < n_part; c0 += 8) {
       Partial q[8];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) q[c] = pr[min(c0 + c, n_chunks - 1)];
+      for (int c = 0; c < 8; ++c) q[c] = pr[min(c0 + c, n_part - 1)];
 #pragma unroll
       for (int c = 0; c < 8; ++c)
-        if (c0 + c < n_chunks) p = merge(p, q[c]);
+        if (c0 + c < n_part) p = merge(p, q[c]);
     }
     if (mj) {
       const float inv = 1.f / p.s;                     // largest probability = 1 / sum exp(x - max)
