@@ -213,7 +213,10 @@ ssm_status ssm_select_build_step_input_varlen(const ssm_step_problem* problems, 
  * keys [cache rows; new rows].  Q^ = RoPE(q, pos), new keys are RoPE(k_new,
  * pos); cached keys are used as given (already rotated at their own positions).
  * RoPE: rotate-half pairs (i, i + d/2), angle pos * theta^(-2i/d); theta == 0
- * disables it.  GQA: query head h reads key/value head h / (h_q / h_kv).
+ * disables it.  The angle is taken modulo one turn in 0.64 fixed point (exact to
+ * below 2^-33 turns for any int32 position), its sine and cosine in fp32, the
+ * rotation in fp32 and rounded to bf16 before the tensor-core products.
+ * GQA: query head h reads key/value head h / (h_q / h_kv).
  * bf16 inputs, fp32 accumulation (tcgen05 tensor cores), bf16 output.
  *
  *   q            bf16 [batch, n_new, h_q, d]
@@ -316,7 +319,8 @@ ssm_status ssm_attention_varlen_core(const void* q, const void* k_new, const voi
  *            (p2 may be NULL unless mode == MARGIN)
  *   commit   uint8 [batch, block_len]
  *   workspace >= ssm_unmask_workspace_size(batch, block_len, vocab, dtype) bytes,
- *            256-byte aligned (per-chunk partial reductions).
+ *            256-byte aligned (the partial reductions of each row: one per
+ *            streaming range of the vocabulary that meets the row).
  * block_len <= 1024. */
 size_t ssm_unmask_workspace_size(int32_t batch, int32_t block_len, int64_t vocab, ssm_dtype dtype);
 
