@@ -960,9 +960,8 @@ ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cud
       return SSM_ERR_CUDA;
     attr_set.fetch_or(bit);
   }
-  ssm::launch_k(attn_fwd_kernel<D, PACKABLE, POLL>, dim3(grid), dim3(kAttnThreads), L::ALLOC, st,
-           m.q128, m.kc, m.vc, m.kn, m.vn, m.kc128, m.vc128,
-                                                                     m.kn128, m.vn128, p);
+  ssm::launch_k(attn_fwd_kernel<D, PACKABLE, POLL>, dim3(grid), dim3(kAttnThreads), L::ALLOC, st, m.q128, m.kc, m.vc,
+                m.kn, m.vn, m.kc128, m.vc128, m.kn128, m.vn128, p);
   return launch_status();
 }
 

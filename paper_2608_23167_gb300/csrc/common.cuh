@@ -82,4 +82,24 @@ inline void launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
   cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // errors: read by launch_status()
 }
 
+// launch_k with programmatic dependent launch also while the stream is being captured (a
+// programmatic edge in the graph).  Used for the unmasking's commit kernel, whose few small CTAs
+// start beside the stream kernel's; the same edge in front of the attention forward and of the
+// unmasking's stream kernel made the graph-replayed step slower (the long sweep 503 -> 541 us).
+template <typename... KArgs, typename... Args>
+inline void launch_k_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                         Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);  // errors: read by launch_status()
+}
+
 }  // namespace ssm

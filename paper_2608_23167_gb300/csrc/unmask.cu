@@ -536,21 +536,9 @@ ssm_status ssm_unmask(const void* logits, ssm_dtype dtype, int32_t batch, int32_
   // being captured (a programmatic edge in the graph): its few small CTAs fit beside the stream
   // kernel's, so its launch and CTA start overlap the stream kernel's tail; its griddepcontrol
   // wait still orders every read after the stream kernel's partials.
-  {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(batch);
-    cfg.blockDim = dim3(threads);
-    cfg.dynamicSmemBytes = shm;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, ssm::unmask_commit_kernel, block_len, plan.n_stage, plan.per, plan.kr, masked,
-                       static_cast<const ssm::Partial*>(part), static_cast<int>(mode), threshold, topk, min_commit,
-                       conf, argmax, p2, commit);
-  }
+  ssm::launch_k_pdl(ssm::unmask_commit_kernel, dim3(batch), dim3(threads), shm, st, block_len, plan.n_stage,
+                    plan.per, plan.kr, masked, static_cast<const ssm::Partial*>(part), static_cast<int>(mode),
+                    threshold, topk, min_commit, conf, argmax, p2, commit);
   return ssm::launch_status();
 }
 
