@@ -61,7 +61,7 @@ __device__ __forceinline__ float words_max(const uint32_t (&w)[16]) {
 // list of its 8 best (value, id) among their entries >= T; each warp then takes
 // its k best by k rounds of warp argmax and one thread merges the eight lists.
 template <typename T>
-__global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restrict__ logits, int64_t vocab,
+__global__ void __launch_bounds__(kTopThreads, 5) topk_row_kernel(const T* __restrict__ logits, int64_t vocab,
                                                               int64_t n_rows, int k, int32_t* __restrict__ ids,
                                                               float* __restrict__ probs) {
   pdl_enter();
@@ -74,9 +74,11 @@ __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restri
   // [chunk][thread] slice maxima, stored in the logits' own type (exact)
   using Slice = typename std::conditional<ESZ == 2, uint16_t, uint32_t>::type;
   Slice* slice_max = reinterpret_cast<Slice*>(ring + kTopStages * kTopStageBytes);
-  __shared__ float red_m[kTopThreads / 32], red_s[kTopThreads / 32];
-  __shared__ float red_kv[(kTopThreads / 32) * kTopMax];
-  __shared__ int red_ki[(kTopThreads / 32) * kTopMax];
+  // the warps' row states and k-best lists, double-buffered by row parity: warp 0 reads one row's
+  // after the CTA barrier while the other warps go on to the next row, which writes the other set
+  __shared__ float red_m[2][kTopThreads / 32], red_s[2][kTopThreads / 32];
+  __shared__ float red_kv[2][(kTopThreads / 32) * kTopMax];
+  __shared__ int red_ki[2][(kTopThreads / 32) * kTopMax];
   __shared__ uint32_t red_key[(kTopThreads / 32) * kTopMax];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t row_bytes = vocab * ESZ;
@@ -105,7 +107,8 @@ __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restri
   for (int q = 0; q < kTopStages; ++q) issue(q);
 
   int slot = 0;
-  for (int64_t row = blockIdx.x; row < n_rows; row += gridDim.x) {
+  int par = 0;  // the row's buffer set
+  for (int64_t row = blockIdx.x; row < n_rows; row += gridDim.x, par ^= 1) {
     float m = -INFINITY, s = 0.f;
     for (int c = 0; c < nchunk; ++c) {
       cp_async_wait<kTopStages - 1>();
@@ -187,24 +190,56 @@ __global__ void __launch_bounds__(kTopThreads) topk_row_kernel(const T* __restri
 #pragma unroll
     for (int d = 16; d >= 1; d >>= 1) ms_merge(m, s, __shfl_xor_sync(0xffffffffu, m, d), __shfl_xor_sync(0xffffffffu, s, d));
     if (lane == 0) {
-      red_m[warp] = m;
-      red_s[warp] = s;
+      red_m[par][warp] = m;
+      red_s[par][warp] = s;
     }
-    warp_topk<kTopMax>(tv, ti, k, red_kv, red_ki);
+    warp_topk<kTopMax>(tv, ti, k, red_kv[par], red_ki[par]);
     __syncthreads();
-    if (threadIdx.x == 0) {
-      float rm = red_m[0], rs = red_s[0];
-      for (int q = 1; q < kTopThreads / 32; ++q) ms_merge(rm, rs, red_m[q], red_s[q]);
+    if (warp == 0) {
+      // lanes 0..7 merge the eight warps' (max, sum); every lane then holds the row's
+      float rm = lane < kTopThreads / 32 ? red_m[par][lane] : -INFINITY;
+      float rs = lane < kTopThreads / 32 ? red_s[par][lane] : 0.f;
+#pragma unroll
+      for (int d = (kTopThreads / 32) / 2; d >= 1; d >>= 1)
+        ms_merge(rm, rs, __shfl_xor_sync(0xffffffffu, rm, d), __shfl_xor_sync(0xffffffffu, rs, d));
+      rm = __shfl_sync(0xffffffffu, rm, 0);
+      rs = __shfl_sync(0xffffffffu, rs, 0);
       const float inv = 1.f / rs;
-      float bv[kTopMax], best;
-      int bi[kTopMax];
-      merge_warp_lists(red_kv, red_ki, k, best, bv, bi);
+      // the k best of the eight lists: lane l holds entries l and l + 32 of the [warp][kTopMax]
+      // table (entries past a list's k are unused), then k rounds of warp argmax, the winning
+      // entry cleared each round
+      constexpr int NE = (kTopThreads / 32) * kTopMax;
+      static_assert(NE <= 64, "two list entries per lane");
+      const bool u0 = lane % kTopMax < k, u1 = (lane + 32) < NE && (lane + 32) % kTopMax < k;
+      float v0 = u0 ? red_kv[par][lane] : -INFINITY, v1 = u1 ? red_kv[par][lane + 32] : -INFINITY;
+      int i0 = u0 ? red_ki[par][lane] : INT_MAX, i1 = u1 ? red_ki[par][lane + 32] : INT_MAX;
       for (int r = 0; r < k; ++r) {
-        ids[row * k + r] = bi[r];
-        probs[row * k + r] = ex2t((bv[r] - rm) * kLog2eT) * inv;
+        const bool first = better(v0, i0, v1, i1) || !(better(v1, i1, v0, i0));
+        float bv = first ? v0 : v1;
+        int bi = first ? i0 : i1;
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) {
+          const float ov = __shfl_xor_sync(0xffffffffu, bv, d);
+          const int oi = __shfl_xor_sync(0xffffffffu, bi, d);
+          if (better(ov, oi, bv, bi)) {
+            bv = ov;
+            bi = oi;
+          }
+        }
+        // ids are distinct within a row, so exactly one entry holds the winner
+        if (i0 == bi) {
+          v0 = -INFINITY;
+          i0 = INT_MAX;
+        } else if (i1 == bi) {
+          v1 = -INFINITY;
+          i1 = INT_MAX;
+        }
+        if (lane == 0) {
+          ids[row * k + r] = bi;
+          probs[row * k + r] = ex2t((bv - rm) * kLog2eT) * inv;
+        }
       }
     }
-    __syncthreads();
   }
   cp_async_wait<0>();
 }

@@ -1,7 +1,6 @@
-// topk.cuh -- pieces of the suffix top-k (the k most probable tokens of a row and
-// their full-vocabulary probabilities, Sec. 3.2 "Soft Suffix Embedding Mixing")
-// shared by the standalone pass (topk.cu) and the fused logits pass (logits.cu):
-// per-thread decreasing candidate lists, the warp and CTA merges of those lists,
+// topk.cuh -- pieces of the suffix top-k pass (topk.cu: the k most probable tokens
+// of a row and their full-vocabulary probabilities, Sec. 3.2 "Soft Suffix Embedding
+// Mixing"): per-thread decreasing candidate lists, the warp merge of those lists,
 // the CTA-wide k-th largest of the threads' maxima, and the (max, sum) merge.
 #pragma once
 
@@ -87,43 +86,6 @@ __device__ __forceinline__ void warp_topk(const float (&lv)[L], const int (&li)[
       ci[L - 1] = INT_MAX;
     }
   }
-}
-
-// The k best of the eight warps' lists in wv / wi (k rounds over their heads);
-// returns the k-th value, sets top to the best one and, if out_v is given,
-// writes the k (value, id).
-__device__ __forceinline__ float merge_warp_lists(const float* wv, const int* wi, int k, float& top, float* out_v,
-                                                  int* out_i) {
-  int head[kTopThreads / 32];
-#pragma unroll
-  for (int w = 0; w < kTopThreads / 32; ++w) head[w] = 0;
-  float t = -INFINITY;
-  for (int r = 0; r < k; ++r) {
-    int bw = 0;
-    float bv = -INFINITY;
-    int bi = INT_MAX;
-#pragma unroll
-    for (int w = 0; w < kTopThreads / 32; ++w) {
-      if (head[w] < k) {
-        const float v = wv[w * kTopMax + head[w]];
-        const int i = wi[w * kTopMax + head[w]];
-        if (better(v, i, bv, bi)) {
-          bv = v;
-          bi = i;
-          bw = w;
-        }
-      }
-    }
-#pragma unroll
-    for (int w = 0; w < kTopThreads / 32; ++w) head[w] += (w == bw) ? 1 : 0;
-    if (out_v) {
-      out_v[r] = bv;
-      out_i[r] = bi;
-    }
-    if (r == 0) top = bv;
-    t = bv;
-  }
-  return t;
 }
 
 __device__ __forceinline__ void ms_merge(float& m, float& s, float m2, float s2) {
