@@ -213,9 +213,10 @@ ssm_status ssm_select_build_step_input_varlen(const ssm_step_problem* problems, 
  * keys [cache rows; new rows].  Q^ = RoPE(q, pos), new keys are RoPE(k_new,
  * pos); cached keys are used as given (already rotated at their own positions).
  * RoPE: rotate-half pairs (i, i + d/2), angle pos * theta^(-2i/d); theta == 0
- * disables it.  The angle is taken modulo one turn in 0.64 fixed point (exact to
- * below 2^-33 turns for any int32 position), its sine and cosine in fp32, the
- * rotation in fp32 and rounded to bf16 before the tensor-core products.
+ * disables it.  The angle pos * f (f the fp64 frequency) is taken modulo one
+ * turn in 0.64 fixed point (exact to below 2^-33 turns for any int32 position),
+ * its sine and cosine in fp32, the rotation in fp32 and rounded to bf16 before
+ * the tensor-core products.
  * GQA: query head h reads key/value head h / (h_q / h_kv).
  * bf16 inputs, fp32 accumulation (tcgen05 tensor cores), bf16 output.
  *

@@ -17,12 +17,12 @@ __device__ __forceinline__ uint32_t rope_pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
-// The D/2 rotation frequencies theta^(-2i/D) (radians per position; all 0 when
-// theta == 0: no rotation), each held as turns per position in 0.64 fixed point:
-// turn_i = round(2^64 * theta^(-2i/D) / (2 pi)).  A position's angle modulo one
-// turn is then the wrapping 64-bit product pos * turn_i, exact up to pos units in
-// the last place (< 2^-33 turns for any int32 position), with no fp64 arithmetic
-// on the device: GB300's fp64 rate is a small fraction of its fp32 rate, and an
+// The D/2 rotation frequencies f_i = theta^(-2i/D) (radians per position, formed
+// in fp64; all 0 when theta == 0: no rotation), each held as turns per position in
+// 0.64 fixed point: turn_i = round(2^64 * f_i / (2 pi)).  A position's angle
+// pos * f_i modulo one turn is then the wrapping 64-bit product pos * turn_i,
+// exact up to pos units in the last place (< 2^-33 turns for any int32 position),
+// with no fp64 arithmetic on the device: GB300's fp64 rate is a small fraction of its fp32 rate, and an
 // fp64 range reduction per angle (and an fp64 exponential and logarithm per
 // table entry) was a visible part of the pre-pass.  Formed on the host once per
 // launch and passed to the kernels by value.
