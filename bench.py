@@ -755,14 +755,21 @@ def time_next_rows(inp: "StepInputs", attn_ms: float, dev, hbm_peak: float, tens
                                               workspace=inp.unmask_ws)
     ms_lp = _event_ms(logits_pass, reps=10)
     lp_bytes = inp.unmask_bytes() + nbytes
-    step_ms = _event_ms(lambda: inp.step(unmask=logits_pass), reps=20)
+    eager_ms = _event_ms(lambda: inp.step(unmask=logits_pass), reps=20)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        inp.step(unmask=logits_pass)
+    torch.cuda.synchronize()
+    step_ms = _event_ms(graph.replay, reps=20)
+    del graph
     out["step_with_suffix_topk"] = {
         "value": inp.n / (step_ms * 1e-3), "unit": UNIT, "ms_per_step": step_ms,
+        "eager_value": inp.n / (eager_ms * 1e-3), "eager_ms_per_step": eager_ms,
         "logits_ms": ms_lp, "logits_GBps": lp_bytes / (ms_lp * 1e-3) / 1e9,
         "logits_frac_hbm": lp_bytes / (ms_lp * 1e-3) / 1e9 / hbm_peak,
-        "how": "the step (eager calls, back to back) with ssm_unmask_topk over the block rows' and the retained "
-               "suffix rows' logits in place of ssm_unmask; logits_* is that call alone (its bytes: both sets of "
-               "logits, read once)"}
+        "how": "the step with ssm_unmask_topk over the block rows' and the retained suffix rows' logits in place "
+               "of ssm_unmask, captured once in a CUDA graph and replayed back to back (eager_*: the same step as "
+               "direct calls); logits_* is that call alone (its bytes: both sets of logits, read once)"}
     del lg, ids, pr
     n = 8192
     kn = W.draw_normal_bf16((1, n, w.h_kv, w.head_dim), 1.0, 71).to(dev)
