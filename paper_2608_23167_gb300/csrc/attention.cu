@@ -287,7 +287,12 @@ struct Unit {
   int64_t orow0;  // packed row of the unit's first query: query = packed / grp, head-in-group = packed % grp
   int64_t qrow0;  // ragged batches: its row in the kv head's block of the rotated queries
   bool two, valid, packed;
+  bool dual;      // two kv heads (g, g + 1) of one problem, one query tile each: slot X takes head g + X
 };
+
+// Ring entries (K or V tiles) a unit streams: its key tiles, twice over for a dual-head unit
+// (entry e is key tile e / 2 of head g + e % 2, so the slots' tiles alternate in the rings).
+__device__ __forceinline__ int unit_entries(const struct Unit& w) { return w.dual ? 2 * w.nt : w.nt; }
 
 // Units are dealt to the persistent CTAs in waves of gridDim.x, each wave in the opposite
 // direction to the last ("snake" order): with units sorted by decreasing cost, a CTA that took
@@ -324,6 +329,8 @@ __device__ __forceinline__ UnitPlan read_plan(const AttnParams& p) {
   return up;
 }
 
+// DUAL = false compiles out the dual-head units (the packable form of the kernel never takes them).
+template <bool DUAL>
 __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& up, int u) {
   Unit w;
   if (up.packed) {
@@ -344,6 +351,22 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
     w.valid = true;
     w.two = pu.rows > kBM;
     w.packed = true;
+    w.dual = false;
+  } else if (DUAL && p.dual_heads) {
+    // two kv heads of one problem, one query tile each (the host takes this form only when every
+    // problem's query rows fit one tile and h_kv is even)
+    const int hp = p.h_kv / 2;
+    w.prob = u / hp;
+    w.g = 2 * (u - w.prob * hp);
+    w.gm = problem_geom(p, w.prob);
+    w.qt0 = 0;
+    w.urows = w.gm.n_new * p.grp;
+    w.orow0 = w.gm.new_row * p.grp;
+    w.qrow0 = w.orow0;
+    w.valid = w.urows > 0;
+    w.two = false;
+    w.packed = false;
+    w.dual = true;
   } else {
     const int pg = u / p.units_per_pg;
     const int pair = u - pg * p.units_per_pg;
@@ -359,6 +382,7 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
     w.valid = w.qt0 < n_qt;
     w.two = p.tiles_per_unit == 2 && w.qt0 + 1 < n_qt;
     w.packed = false;
+    w.dual = false;
   }
   w.n_csub = (w.gm.n_cache + kSub - 1) / kSub;
   w.n_nsub = (w.gm.n_new + kSub - 1) / kSub;
@@ -366,7 +390,9 @@ __device__ __forceinline__ Unit make_unit(const AttnParams& p, const UnitPlan& u
   return w;
 }
 
-template <int D, bool PACKABLE, bool POLL>
+// DUAL compiles the dual-head units in (only without packed units): a separate form, so that the
+// other forms carry none of their code.
+template <int D, bool PACKABLE, bool POLL, bool DUAL>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
     const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kn,
@@ -441,20 +467,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int fills = 0;   // tiles loaded into this ring so far (all units)
       const int nst = half ? kVStages : kKStages;
       for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
-        const Unit w = make_unit(p, up, u);
+        const Unit w = make_unit<DUAL>(p, up, u);
         if (!w.valid) continue;
         if (!half) {
           if (qcount > 0) ok = warp_wait<POLL>(&bars[Q_EMPTY], (qcount - 1) & 1, p.wait_ns);
           if (!ok) break;
-          const int nq = w.two ? 2 : 1;
+          const int nq = (w.two || w.dual) ? 2 : 1;
           mbar_arrive_expect_tx_if(leader, &bars[Q_FULL], nq * L::TILE);
           for (int x = 0; x < nq; ++x) {
+            // a pair: tiles qt0 and qt0 + 1 of kv head g; dual heads: tile qt0 of heads g and g + 1
+            const int gx = w.g + (w.dual ? x : 0);
+            const int tx = w.dual ? 0 : x;
             int qy, qz;
             if (uniform) {
-              qy = (w.qt0 + x) * kBM;
-              qz = w.prob * p.h_kv + w.g;
+              qy = (w.qt0 + tx) * kBM;
+              qz = w.prob * p.h_kv + gx;
             } else {
-              qy = static_cast<int>(static_cast<int64_t>(w.g) * p.qrows_g + w.qrow0) + x * kBM;
+              qy = static_cast<int>(static_cast<int64_t>(gx) * p.qrows_g + w.qrow0) + tx * kBM;
               qz = 0;
             }
 #pragma unroll
@@ -465,7 +494,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           ++qcount;
         }
         const int c3 = uniform ? w.prob : 0;
-        for (int jt = 0; jt < w.nt && ok; ++jt) {
+        const int ne = unit_entries(w);
+        for (int e = 0; e < ne && ok; ++e) {
+          const int jt = w.dual ? (e >> 1) : e;            // key tile
+          const int gh = w.g + (w.dual ? (e & 1) : 0);     // its kv head
           const int st = fills % nst, fill = fills / nst;
           if (fill > 0) ok = warp_wait<POLL>(&bars[(half ? V_EMPTY : K_EMPTY) + st], (fill - 1) & 1, p.wait_ns);
           if (!ok) break;
@@ -481,7 +513,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
                                        : (uniform ? (sub0 - w.n_csub) * kSub
                                                   : static_cast<int>(w.gm.new_row + (sub0 - w.n_csub) * kSub));
 #pragma unroll
-            for (int pn = 0; pn < NP; ++pn) tma_load_4d_if(leader, dst + pn * kPanel, map, full, pn * 64, w.g, c2, c3);
+            for (int pn = 0; pn < NP; ++pn) tma_load_4d_if(leader, dst + pn * kPanel, map, full, pn * 64, gh, c2, c3);
           } else {
 #pragma unroll
             for (int sb = 0; sb < 4; ++sb) {
@@ -500,7 +532,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
               }
 #pragma unroll
               for (int pn = 0; pn < NP; ++pn)
-                tma_load_4d_if(leader, dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, w.g, c2, c3);
+                tma_load_4d_if(leader, dst + pn * kPanel + sb * kSub * 128, map, full, pn * 64, gh, c2, c3);
             }
           }
           ++fills;
@@ -528,7 +560,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       int kbase = 0, vbase = 0;  // global index of the unit's first K / V tile
       int pv0 = 0, pv1 = 0;      // PV GEMMs issued per slot (all units)
       for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
-        const Unit w = make_unit(p, up, u);
+        const Unit w = make_unit<DUAL>(p, up, u);
         if (!w.valid) continue;
         ok = warp_wait<POLL>(&bars[Q_FULL], ucount & 1, p.wait_ns);
         if (!ok) break;
@@ -563,12 +595,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
           ++pv;
           return true;
         };
-        const int n_jobs = w.two ? 2 * w.nt : w.nt;
+        // jobs alternate between the slots; j is the job's ring entry (a pair shares each entry)
+        const int n_jobs = w.two ? 2 * w.nt : unit_entries(w);
         for (int t = 0; t < n_jobs && ok; ++t) {
           const int x = t & 1;
           const int j = w.two ? (t >> 1) : t;
           const int ki = kbase + j;
-          const uint64_t qb = dQ + static_cast<uint64_t>(((w.two ? x : 0) * L::TILE) >> 4);
+          const uint64_t qb = dQ + static_cast<uint64_t>((((w.two || w.dual) ? x : 0) * L::TILE) >> 4);
           const uint64_t kb = dK + static_cast<uint64_t>(((ki % kKStages) * L::TILE) >> 4);
           const uint32_t s_tmem = tmem + x * kBN;
           if ((x ? kx1 : kx0) > 0) {
@@ -593,8 +626,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         if (ok && kx0 > 0) ok = issue_pv(0);
         if (ok && kx1 > 0) ok = issue_pv(1);
         if (ok) ok = wait_o_free(0) && wait_o_free(1);
-        kbase += w.nt;
-        vbase += w.nt;
+        kbase += unit_entries(w);
+        vbase += unit_entries(w);
         ++ucount;
       }
       if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
@@ -638,10 +671,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         return true;
       };
       for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
-        const Unit w = make_unit(p, up, u);
+        const Unit w = make_unit<DUAL>(p, up, u);
         if (!w.valid) continue;
         int kx0 = 0, kx1 = 0, jlast0 = 0, jlast1 = 0;
-        const int n_jobs = w.two ? 2 * w.nt : w.nt;
+        const int n_jobs = w.two ? 2 * w.nt : unit_entries(w);
         for (int t = 0; t < n_jobs && ok; ++t) {
           const int x = t & 1;
           const int j = w.two ? (t >> 1) : t;
@@ -650,7 +683,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         }
         if (ok && kx0 > 0) ok = vouch(0, jlast0, -1);
         if (ok && kx1 > 0) ok = vouch(1, jlast1, -1);
-        kbase += w.nt;
+        kbase += unit_entries(w);
       }
       if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
     }
@@ -668,9 +701,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
     int sj = 0;       // S tiles consumed by this slot (all units)
     int merges = 0;   // split-key merges done
     for (int k_u = 0, u = snake_unit(0); u < up.total_units && ok; u = snake_unit(++k_u)) {
-      const Unit w = make_unit(p, up, u);
+      const Unit w = make_unit<DUAL>(p, up, u);
       if (!w.valid) continue;
-      const int jobs = w.two ? w.nt : (x == 0 ? (w.nt + 1) / 2 : w.nt / 2);
+      const int jobs = (w.two || w.dual) ? w.nt : (x == 0 ? (w.nt + 1) / 2 : w.nt / 2);
       float m_run = -INFINITY, l_run = 0.f;
       // this thread's query row within the unit; with packed units, its own problem's keys:
       // cache rows below lim, new rows [nlo, nhi) (rows past the unit's end see every key;
@@ -686,7 +719,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         nhi = mine ? bd.z - static_cast<int>(w.gm.new_row) : nhi;
       }
       for (int k = 0; k < jobs; ++k) {
-        const int j = w.two ? k : 2 * k + x;
+        const int j = (w.two || w.dual) ? k : 2 * k + x;
         // The tile's masking plan is made while the tensor core still computes S (it depends
         // only on the tile index and the row's bounds): valid keys of each 32-key sub-box of
         // the tile for this row, columns [lo, hi)
@@ -815,7 +848,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
       // The buffer is rewritten only after slot B's last PV of a later unit, which the MMA
       // issues after slot A freed this unit's accumulators, i.e. after slot A's reads.
       float mB = -INFINITY, lB = 0.f;
-      if (!w.two && w.nt >= 2) {
+      const bool split = !w.two && !w.dual && w.nt >= 2;   // the slots split the key tiles
+      if (split) {
         if (x == 1) {
           merge_buf[row] = m_run;
           merge_buf[kBM + row] = l_run;
@@ -828,11 +862,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         }
         ++merges;
       }
-      if (w.two || x == 0) {
+      if (w.two || w.dual || x == 0) {
         const bool valid = pr_u < w.urows;
         const int64_t prow = w.orow0 + pr_u;    // packed (query, head-in-group) row
         const int64_t qrow = prow / p.grp;      // the query's new row
-        const int h = w.g * p.grp + static_cast<int>(prow - qrow * p.grp);
+        const int h = (w.g + (w.dual ? x : 0)) * p.grp + static_cast<int>(prow - qrow * p.grp);
         const float m = fmaxf(m_run, mB);
         const float ea = ex2_approx(m_run - m), eb = ex2_approx(mB - m);
         const float a = (l_run > 0.f) ? ea : 0.f;
@@ -859,7 +893,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
             for (int v = 0; v < 4; ++v) st_global_v4_pred(d4 + v, v4[v], valid);
           }
         };
-        if (!w.two && w.nt >= 2) {
+        if (split) {
           // split keys: both accumulators, 64 columns at a time, each pair of loads one round trip
           // (warp-uniform; cb = 0 for a row slot B gave no weight)
 #pragma unroll
@@ -892,7 +926,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_fwd_kernel(
         // this slot's O (and, with split keys, slot B's O too) may now be overwritten
         tc_fence_before_sync();
         warp_arrive(&bars[O_FREE + x]);
-        if (!w.two) warp_arrive(&bars[O_FREE + 1]);
+        if (!w.two && !w.dual) warp_arrive(&bars[O_FREE + 1]);
       }
     }
     if (!ok) record_error(p.err, SSM_ERR_TIMEOUT);
@@ -966,14 +1000,14 @@ WsLayout ws_layout(int64_t total_new, int32_t h_q, int32_t h_kv, int32_t d) {
 
 // One instantiation of the forward: the register split assumes the compiled register count
 // (checked once), the dynamic shared memory is opted into once per device.
-template <int D, bool PACKABLE, bool POLL>
+template <int D, bool PACKABLE, bool POLL, bool DUAL>
 ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
   using L = Layout<D>;
   static std::atomic<int> regs_ok{0};  // 0 unknown, 1 ok, 2 mismatch
   int st_regs = regs_ok.load();
   if (st_regs == 0) {
     cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, PACKABLE, POLL>) != cudaSuccess) return SSM_ERR_CUDA;
+    if (cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, PACKABLE, POLL, DUAL>) != cudaSuccess) return SSM_ERR_CUDA;
     st_regs = fa.numRegs == kLaunchRegs ? 1 : 2;
     regs_ok.store(st_regs);
   }
@@ -983,12 +1017,12 @@ ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cud
   if (cudaGetDevice(&dev) != cudaSuccess) return SSM_ERR_CUDA;
   const uint64_t bit = 1ull << (dev & 63);
   if (!(attr_set.load() & bit)) {
-    if (cudaFuncSetAttribute(attn_fwd_kernel<D, PACKABLE, POLL>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
+    if (cudaFuncSetAttribute(attn_fwd_kernel<D, PACKABLE, POLL, DUAL>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC) !=
         cudaSuccess)
       return SSM_ERR_CUDA;
     attr_set.fetch_or(bit);
   }
-  ssm::launch_k(attn_fwd_kernel<D, PACKABLE, POLL>, dim3(grid), dim3(kAttnThreads), L::ALLOC, st, m.q128, m.kc, m.vc,
+  ssm::launch_k(attn_fwd_kernel<D, PACKABLE, POLL, DUAL>, dim3(grid), dim3(kAttnThreads), L::ALLOC, st, m.q128, m.kc, m.vc,
                 m.kn, m.vn, m.kc128, m.vc128, m.kn128, m.vn128, p);
   return launch_status();
 }
@@ -998,8 +1032,12 @@ ssm_status launch_fwd_form(const AttnMaps& m, const AttnParams& p, int grid, cud
 // form with blocking probes.
 template <int D, bool PACKABLE>
 ssm_status launch_fwd(const AttnMaps& m, const AttnParams& p, int grid, cudaStream_t st) {
-  if (p.wait_ns < kPollLimitNs) return launch_fwd_form<D, PACKABLE, true>(m, p, grid, st);
-  return launch_fwd_form<D, PACKABLE, false>(m, p, grid, st);
+  if (!PACKABLE && p.dual_heads) {
+    if (p.wait_ns < kPollLimitNs) return launch_fwd_form<D, false, true, true>(m, p, grid, st);
+    return launch_fwd_form<D, false, false, true>(m, p, grid, st);
+  }
+  if (p.wait_ns < kPollLimitNs) return launch_fwd_form<D, PACKABLE, true, false>(m, p, grid, st);
+  return launch_fwd_form<D, PACKABLE, false, false>(m, p, grid, st);
 }
 
 template <int D>
@@ -1101,9 +1139,18 @@ ssm_status launch_attention(const void* q, const void* k_new, const void* v_new,
     const int64_t pair_cost = ((pgs * ((m_tiles + 1) / 2) + sms - 1) / sms) * nt;
     const int64_t single_cost = ((pgs * m_tiles + sms - 1) / sms) * ((nt + 1) / 2 + 1);
     p.tiles_per_unit = single_cost < pair_cost ? 1 : 2;
+    // Problems of one query tile whose single-tile units take more than one round: units of two
+    // kv heads (one tile each, each slot on its own head's key tiles) halve the unit count; a
+    // unit's chain is then all its key tiles, both slots streaming at once.
+    p.dual_heads = 0;
+    if (!may_pack && m_tiles == 1 && h_kv % 2 == 0) {
+      const int64_t dual_cost = ((pgs / 2 + sms - 1) / sms) * nt;
+      if (dual_cost < single_cost) p.dual_heads = 1;
+    }
   }
   p.units_per_pg = p.tiles_per_unit == 2 ? (m_tiles + 1) / 2 : m_tiles;
-  const int64_t total_units = static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
+  const int64_t total_units =
+      p.dual_heads ? static_cast<int64_t>(n_prob) * (h_kv / 2) : static_cast<int64_t>(p.units_per_pg) * n_prob * h_kv;
   if (total_units > INT32_MAX) return SSM_ERR_UNSUPPORTED;
   p.total_units = static_cast<int32_t>(total_units);
   if (!may_pack) return launch_fwd<D, false>(m, p, static_cast<int>(std::min<int64_t>(total_units, num_sms())), st);

@@ -61,6 +61,7 @@ struct AttnParams {
   int4* row_bounds;                  // ragged batches: per new row, its problem's (n_cache, new_row, new_row + n_new)
   int32_t units_per_pg;              // work units per (problem, kv head)
   int32_t tiles_per_unit;            // problem units: 128-row query tiles per unit (2: a pair, 1: single tiles)
+  int32_t dual_heads;                // problem units of one query tile: two kv heads of one problem per unit
   int32_t total_units;
   float scale_log2;                  // softmax scale * log2(e)
   __nv_bfloat16* out;

@@ -25,13 +25,14 @@ def dev():
     return cuda_or_skip()
 
 
-@pytest.mark.parametrize("shape", ["two_tiles", "split_keys"])
+@pytest.mark.parametrize("shape", ["two_tiles", "dual_heads", "split_keys"])
 def test_attention_wait_timeout_reports_and_recovers(dev, shape):
     """two_tiles: one 589-row problem without cache (units of two query tiles, 32 heads);
-    split_keys: 8 sequences x 101 rows over 512-row caches (one query tile per unit: the two
+    dual_heads: 8 sequences x 101 rows over 512-row caches, 32 heads (units of two kv heads,
+    one query tile each); split_keys: the same with 8 heads (one query tile per unit: the two
     softmax slots split the key tiles and meet at the merge wait)."""
     from paper_2608_23167_gb300 import ssm
-    h, d = 32, 128
+    h, d = (8 if shape == "split_keys" else 32), 128
     sizes = [(589, 0)] if shape == "two_tiles" else [(101, 512)] * 8
     rows, new_row = [], 0
     for i, (n, c) in enumerate(sizes):
