@@ -75,6 +75,11 @@ __device__ __forceinline__ void zero_row(uint4* __restrict__ dst, int hvec) {
   for (int v = threadIdx.x; v < hvec; v += kBuildThreads) dst[v] = make_uint4(0, 0, 0, 0);
 }
 
+// COLS: 16-byte columns of a retained suffix row each thread gathers per pass, with every load
+// of the pass in flight (one pass of the row per COLS * kBuildThreads columns).  Two columns
+// halve a hidden-4096 row's memory round trips but take 88 registers against 52 (five CTAs
+// per SM instead of nine): the host takes them for small launches (two_columns below).
+template <int COLS>
 __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const BuildParams p) {
   pdl_enter();
   __shared__ int32_t s_ids[kMaxK];
@@ -194,15 +199,15 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
     return;
   }
   const float keep = 1.f - p.alpha;
-  for (int v = threadIdx.x; v < p.hvec; v += kBuildThreads) {
-    float acc[8];
-    {
+  // gather the candidate rows six at a time: all of a chunk's loads (and the [MASK] row's) for
+  // the pass's COLS columns are in flight together; the products are added in candidate order
+  constexpr int C = 6;
+  if constexpr (COLS == 1) {
+    for (int v = threadIdx.x; v < p.hvec; v += kBuildThreads) {
+      float acc[8];
       const uint4 mv = __ldg(e_mask + v);
 #pragma unroll
       for (int c = 0; c < 8; ++c) acc[c] = 0.f;
-      // gather the candidate rows six at a time: all of a chunk's loads (and the [MASK]
-      // row's) are in flight together; the products are added in candidate order
-      constexpr int C = 6;
       for (int j = 0; j < n; j += C) {
         uint4 ev[C];
 #pragma unroll
@@ -223,15 +228,75 @@ __global__ void __launch_bounds__(kBuildThreads) build_step_input_kernel(const B
       unpack8(mv, m);
 #pragma unroll
       for (int c = 0; c < 8; ++c) acc[c] = fmaf(keep, m[c], acc[c]);
+      uint4 o;
+      o.x = pack2(acc[0], acc[1]);
+      o.y = pack2(acc[2], acc[3]);
+      o.z = pack2(acc[4], acc[5]);
+      o.w = pack2(acc[6], acc[7]);
+      dst[v] = o;
     }
-    uint4 o;
-    o.x = pack2(acc[0], acc[1]);
-    o.y = pack2(acc[2], acc[3]);
-    o.z = pack2(acc[4], acc[5]);
-    o.w = pack2(acc[6], acc[7]);
-    dst[v] = o;
+    return;
+  }
+  for (int v0 = threadIdx.x; v0 < p.hvec; v0 += COLS * kBuildThreads) {
+    bool on[COLS];
+    float acc[COLS][8];
+    uint4 mv[COLS];
+#pragma unroll
+    for (int q = 0; q < COLS; ++q) {
+      on[q] = v0 + q * kBuildThreads < p.hvec;
+      mv[q] = on[q] ? __ldg(e_mask + v0 + q * kBuildThreads) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[q][c] = 0.f;
+    }
+    for (int j = 0; j < n; j += C) {
+      uint4 ev[COLS][C];
+#pragma unroll
+      for (int u = 0; u < C; ++u) {
+        if (j + u < n) {
+          const uint4* rowp = p.embed + static_cast<int64_t>(s_ids[j + u]) * p.hvec + v0;
+#pragma unroll
+          for (int q = 0; q < COLS; ++q)
+            if (on[q]) ev[q][u] = __ldg(rowp + q * kBuildThreads);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < C; ++u) {
+        if (j + u < n) {
+          const float w = s_w[j + u];
+#pragma unroll
+          for (int q = 0; q < COLS; ++q) {
+            if (on[q]) {
+              float f[8];
+              unpack8(ev[q][u], f);
+#pragma unroll
+              for (int c = 0; c < 8; ++c) acc[q][c] = fmaf(w, f[c], acc[q][c]);
+            }
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < COLS; ++q) {
+      if (!on[q]) continue;
+      float m[8];
+      unpack8(mv[q], m);
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[q][c] = fmaf(keep, m[c], acc[q][c]);
+      uint4 o;
+      o.x = pack2(acc[q][0], acc[q][1]);
+      o.y = pack2(acc[q][2], acc[q][3]);
+      o.z = pack2(acc[q][4], acc[q][5]);
+      o.w = pack2(acc[q][6], acc[q][7]);
+      dst[v0 + q * kBuildThreads] = o;
+    }
   }
 }
+
+// Small launches take the two-column form: up to about one and a half waves of it (five CTAs per
+// SM at its 88 registers; the serving batch's 808 rows measured 1 us faster with it), where the
+// row's round trips, not the bytes in flight, set the time.  Large launches (the sweep's
+// 11008 CTAs) keep nine CTAs per SM of the one-column form.
+inline bool two_columns(int64_t ctas) { return ctas <= 8ll * num_sms(); }
 
 ssm_status check_common(const void* embed, int64_t vocab, int32_t hidden, int32_t mask_id, int32_t k,
                         float alpha, int32_t block_len, const void* x_out) {
@@ -288,8 +353,12 @@ ssm_status ssm_build_step_input(const int32_t* block_tokens, const int32_t* pref
   p.pos_out = pos_out;
   p.err = ssm::device_error_word();
   dim3 grid(rows, batch);
-  ssm::launch_k(ssm::build_step_input_kernel, dim3(grid), dim3(ssm::kBuildThreads), 0, reinterpret_cast<cudaStream_t>(stream),
-           p);
+  if (ssm::two_columns(static_cast<int64_t>(rows) * batch))
+    ssm::launch_k(ssm::build_step_input_kernel<2>, dim3(grid), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
+  else
+    ssm::launch_k(ssm::build_step_input_kernel<1>, dim3(grid), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
   return ssm::launch_status();
 }
 
@@ -327,8 +396,12 @@ ssm_status ssm_build_step_input_varlen(const ssm_step_problem* problems, int32_t
   p.pos_out = pos_out;
   p.err = ssm::device_error_word();
   dim3 grid(max_rows, n_problems);
-  ssm::launch_k(ssm::build_step_input_kernel, dim3(grid), dim3(ssm::kBuildThreads), 0, reinterpret_cast<cudaStream_t>(stream),
-           p);
+  if (ssm::two_columns(static_cast<int64_t>(max_rows) * n_problems))
+    ssm::launch_k(ssm::build_step_input_kernel<2>, dim3(grid), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
+  else
+    ssm::launch_k(ssm::build_step_input_kernel<1>, dim3(grid), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
   return ssm::launch_status();
 }
 
@@ -365,8 +438,12 @@ ssm_status ssm_select_build_step_input_varlen(const ssm_step_problem* problems, 
   p.x_out = static_cast<uint4*>(x_out);
   p.pos_out = pos_out;
   p.err = ssm::device_error_word();
-  ssm::launch_k(ssm::build_step_input_kernel, dim3(max_rows, n_problems), dim3(ssm::kBuildThreads), 0,
-                reinterpret_cast<cudaStream_t>(stream), p);
+  if (ssm::two_columns(static_cast<int64_t>(max_rows) * n_problems))
+    ssm::launch_k(ssm::build_step_input_kernel<2>, dim3(max_rows, n_problems), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
+  else
+    ssm::launch_k(ssm::build_step_input_kernel<1>, dim3(max_rows, n_problems), dim3(ssm::kBuildThreads), 0,
+                  reinterpret_cast<cudaStream_t>(stream), p);
   return ssm::launch_status();
 }
 
