@@ -213,3 +213,28 @@ def test_unmask_long_sweep_full_size_sampled(dev, mode, threshold, want_p2):
         if want_p2:
             assert np.allclose(p2[s:s + 1].cpu().double().numpy(), p2_r, rtol=1e-5, atol=1e-30), f"sequence {s}"
         _check_commits(conf_r, p2_r, masked[s:s + 1].numpy(), commit[s:s + 1], commit_r, md, threshold, 1, 1)
+
+
+@pytest.mark.parametrize("B,mode,threshold,topk,min_commit", [
+    (64, "threshold", 0.5, 1, 3),     # two warps of positions per sequence
+    (200, "topk", 0.0, 17, 0),        # a ragged last warp
+    (1000, "margin", 0.3, 1, 2),      # close to the 1024-position limit of a block
+])
+def test_unmask_long_blocks(dev, B, mode, threshold, topk, min_commit):
+    """Blocks longer than 32 positions: the commit kernel's CTA has one thread per position
+    (up to 1024), and its ranking runs over every position of the block.  Confidences are
+    planted from 0.02 to 0.95 (at 64 and 200 positions far more than the 1e-3 ranking band
+    apart, so every position is compared exactly; at 1000 positions 9e-4 apart, so the
+    ranking boundary's neighbours are checked as a valid commit set)."""
+    batch, V = 2, 512
+    logits = _separated_logits(batch, B, V, "f32", 7 + B, 0.02, 0.95)
+    g = torch.Generator().manual_seed(B)
+    masked = (torch.rand((batch, B), generator=g) < 0.7).to(torch.uint8)
+    md = MODES[mode]
+    conf, arg, p2, commit = _gpu_unmask(dev, logits, masked, md, threshold, topk, min_commit)
+    conf_r, arg_r, p2_r, commit_r = O.unmask(f64(logits), masked.numpy(), md, threshold, topk, min_commit)
+    m = masked.numpy().astype(bool)
+    assert np.array_equal(arg[m], arg_r[m])
+    assert np.allclose(conf[m], conf_r[m], rtol=1e-5, atol=0)
+    assert np.allclose(p2[m], p2_r[m], rtol=1e-5, atol=1e-30)
+    _check_commits(conf_r, p2_r, masked.numpy(), commit, commit_r, md, threshold, topk, min_commit)
