@@ -99,6 +99,7 @@ def _check_commits(conf_r, p2_r, masked, commit_g, commit_r, mode, threshold, to
     ("f32", 4096, 2, 3.0, 0.3, 0.5),
     ("bf16", 126464, 8, 4.0, 0.25, 1.0),      # serving workload, planted confident rows
     ("bf16", 126464, 2, 4.0, 0.0, 0.5),
+    ("f32", 126464, 2, 4.0, 0.25, 0.8),       # fp32 rows of 31 stages, the last one partial
     ("bf16", 126464, 24, 4.0, 0.25, 0.9),     # 768 rows: a CTA's stage range ends inside rows and spans several
     ("bf16", 8192, 64, 4.0, 0.25, 0.6),       # one-stage rows: a range holds whole rows, masked and not
     ("bf16", 50001, 2, 2.0, 0.5, 0.7),        # odd vocabulary: unaligned rows take the scalar path
