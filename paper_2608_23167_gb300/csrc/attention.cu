@@ -9,10 +9,11 @@
 //    (query i, head-in-group hl) -> row i * grp + hl, so that a 128-row M tile
 //    of the tensor-core GEMM holds every query head that shares a K/V head.
 //  * attn_fwd_kernel: persistent, one CTA per SM.  Work units are (problem,
-//    kv head, pair of 128-row query tiles) or, for ragged batches whose
-//    problems share one cache prefix, pairs of tiles of consecutive problems'
-//    packed rows (each row masked to its own prefix and new rows); they are
-//    dealt in snake order, and barrier phases carry over from unit to unit,
+//    kv head, pair of 128-row query tiles), (problem, kv head, one tile) or
+//    (problem, two kv heads, one tile each), whichever the host's makespan
+//    estimate prefers, or, for ragged batches whose problems share one cache
+//    prefix, pairs of tiles of consecutive problems' packed rows (each row
+//    masked to its own prefix and new rows); they are dealt in snake order, and barrier phases carry over from unit to unit,
 //    so the next unit's Q/K loads and first QK^T overlap the current unit's
 //    last softmax and epilogue.  Per unit,
 //    warps 0 and 2 stream the K and the V tiles with TMA, each ring at its own
@@ -25,7 +26,8 @@
 //    while one turns its S tile into P (written back over S as bf16), the
 //    tensor core runs the other slot's GEMMs.  With two query tiles each slot
 //    owns one; with a single query tile the slots split the key tiles
-//    (even/odd) and merge their partial softmax states at the end.  After a
+//    (even/odd) and merge their partial softmax states at the end; with two
+//    kv heads each slot owns one head's tile and key tiles.  After a
 //    slot's first tile of a unit the exponentials are taken against the
 //    current reference without a row maximum; O is rescaled only when a
 //    tile's row sum of p exceeds 2^16.
